@@ -1,0 +1,358 @@
+"""Throughput of one global round of distributed sign momentum with local steps.
+
+A step is one global round of Algorithm 1 on the synthetic workload: tau
+times (synthetic gradient fill for all n workers + one local base-optimizer
+step on all n replicas), then the fused global step and its statistics.
+All inputs are resident in HBM when the timed region starts.
+
+Metric: params/s per global round = d x rounds / device time (whole job).
+Also reported: the dominant kernel's roofline (algorithmic bytes per launch
+over its CUDA-event duration, against the measured HBM copy bandwidth), an
+end-to-end figure through the C ABI with host gradient buffers, the SM
+clocks seen during the timed region, and the CPU oracle timed on a bounded
+sample of the same workload.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload gpt2s] [--impl reference]
+
+Under torchrun each rank runs its own parameter shard of the workload's size
+(the path is elementwise, so a shard needs no communication); rank 0 prints
+one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "params/s per global round (τ local + sign-momentum step); % HBM roofline"
+UNIT = "params/s"
+CPU_SAMPLE_ELEMS = 1 << 22
+KERNELS_SRC = os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", "dsm_kernels.cu")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default=W.BENCH_WORKLOAD, choices=sorted(W.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def bytes_per_elem_local(wl) -> int:
+    """Algorithmic bytes of one local step per worker-element: every state read and written once."""
+    g = 2 if wl.hp.grad_dtype == W.BF16 else 4
+    if wl.hp.base == W.BASE_ADAMW:
+        return 6 * 4 + g      # read x, m, v, g; write x, m, v
+    return 4 * 4 + g          # read x, buf, g; write x, buf
+
+
+def bytes_per_param_global(wl) -> int:
+    return 8 * (wl.n + 2)     # read x, m and n replicas; write x, m and n replicas
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def committed_traffic(kernel_key):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernels."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        j = json.load(f)
+    src_hash = hashlib.sha256(open(KERNELS_SRC, "rb").read()).hexdigest()[:16]
+    ent = j.get(kernel_key)
+    if not ent or ent.get("kernels_sha256_16") != src_hash:
+        return None
+    return ent.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.proc = None
+        self.gpu = gpu_index
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.3)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.strip().splitlines():
+            f = [c.strip() for c in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(f[1]), max=float(f[2]), power=float(f[3]), hw=f[5], hwt=f[6],
+                                 swt=f[7], pcap=f[8]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        pmax = max(r["power"] for r in rows)
+        loaded = [r for r in rows if r["power"] >= 0.5 * pmax] or rows
+        reasons = set()
+        for r in rows:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in loaded), "sm_max_mhz": rows[0]["max"],
+                "reasons": sorted(reasons), "samples": len(rows), "power_w_max": pmax}
+
+
+def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, rounds=1):
+    """The CPU oracle, as it stands, on one round over a contiguous sample of the workload."""
+    import numpy as np
+
+    from oracle import dsm_oracle as O
+    count = min(elems_count, wl.d)
+    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64))
+    t0 = time.perf_counter()
+    for _ in range(rounds):
+        ora.run_round()
+    dt = time.perf_counter() - t0
+    return {"value": count * rounds / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{rounds} round(s) (tau={wl.tau} local steps x n={wl.n} workers + global step) over "
+                      f"elements [0, {count}) of the {wl.d}-parameter layout, numpy fp32, one thread; "
+                      f"{dt:.2f} s"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    wl = W.WORKLOADS[args.workload]
+    import numpy as np
+
+    from oracle import dsm_oracle as O
+    count = min(1 << 20, wl.d)
+    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64))
+    for _ in range(args.warmup):
+        ora.run_round()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ora.run_round()
+    dt = time.perf_counter() - t0
+    value = count * args.steps / dt
+    sample = (f"each step: one round (tau={wl.tau} x n={wl.n} local steps + global step) over elements "
+              f"[0, {count}) of the {wl.d}-parameter layout; numpy fp32 oracle, one thread")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": workload_config(wl, args.gpus),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(wl, gpus):
+    return {"workload": wl.name, "d": wl.d, "n_workers": wl.n, "tau": wl.tau, "tensors": len(wl.tensors),
+            "base": "adamw" if wl.hp.base == W.BASE_ADAMW else "sgd-momentum",
+            "grad_dtype": "bf16" if wl.hp.grad_dtype == W.BF16 else "f32",
+            "sign": ["sign", "rand-sign-2", "rand-sign-1"][wl.hp.sign_mode],
+            "parallelism": f"param-shard x{gpus}" if gpus > 1 else "single GPU",
+            "l2": "inputs larger than L2 (129 MB): each local-step launch streams "
+                  f"{wl.n * wl.d * bytes_per_elem_local(wl) / 1e9:.1f} GB"}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    rank, world, local = dist_env()
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2411_17866_gb300 import dsm
+    if world > 1:
+        dist.init_process_group("gloo", rank=rank, world_size=world)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = W.WORKLOADS[args.workload]
+    import dataclasses
+    hp = dataclasses.replace(wl.hp, seed=wl.hp.seed + rank)
+    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    tau = wl.tau
+
+    def round_(t, local_events=None, global_events=None):
+        for k in range(tau):
+            run.fill_synthetic_grads(t * tau + k, stream)
+            if local_events is not None:
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                run.local_step(stream)
+                b.record(stream)
+                local_events.append((a, b))
+            else:
+                run.local_step(stream)
+        if global_events is not None:
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            run.global_step(stream)
+            b.record(stream)
+            global_events.append((a, b))
+        else:
+            run.global_step(stream)
+
+    t = 0
+    for _ in range(args.warmup):
+        round_(t)
+        t += 1
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local) if (rank == 0 and not args.no_clocks) else None
+    if sampler:
+        sampler.start()
+    local_ev, global_ev = [], []
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(args.steps):
+        round_(t, local_ev, global_ev)
+        t += 1
+    end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    elapsed = start.elapsed_time(end) / 1e3
+    if world > 1:
+        tt = torch.tensor([elapsed], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed = float(tt.item())
+    local_ms = [a.elapsed_time(b) for a, b in local_ev]
+    global_ms = [a.elapsed_time(b) for a, b in global_ev]
+
+    # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device
+    # gradient copy + local step), the global step, and the new x read back to pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        esz = 2 if wl.hp.grad_dtype == W.BF16 else 4
+        gdt = torch.bfloat16 if esz == 2 else torch.float32
+        host_g = torch.empty((wl.n, wl.d), dtype=gdt).pin_memory()
+        run.fill_synthetic_grads(t * tau, stream)   # the gradients of one synthetic step, staged once
+        for i in range(wl.n):
+            run.read(dsm.BUF_GRAD, i, out=host_g[i], stream=stream)
+        host_x = torch.empty(wl.d, dtype=torch.float32).pin_memory()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            for k in range(tau):
+                run.load_grads(host_g, stream)
+                run.local_step(stream)
+            run.global_step(stream)
+            run.read(dsm.BUF_X, out=host_x, stream=stream)   # synchronises the stream
+            t += 1
+        e2e_dt = time.perf_counter() - t0
+        if world > 1:
+            tt = torch.tensor([e2e_dt], dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_dt = float(tt.item())
+        e2e = {"value": world * wl.d * args.e2e_steps / e2e_dt, "unit": UNIT,
+               "h2d_bytes_per_step": tau * wl.n * wl.d * esz, "d2h_bytes_per_step": wl.d * 4,
+               "steps": args.e2e_steps, "path": "dsm_load_grads (pinned host) + dsm_local_step x tau, "
+                                                 "dsm_global_step, dsm_read_params(x -> pinned host)"}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return 0
+
+    peak, peak_kind = measured_peaks()
+    local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
+    avg_local_s = statistics.mean(local_ms) / 1e3
+    achieved = local_bytes / avg_local_s / 1e9
+    kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
+    traffic = committed_traffic(f"{kname}:{args.workload}")
+    global_bytes = wl.d * bytes_per_param_global(wl)
+    avg_global_s = statistics.mean(global_ms) / 1e3
+    value = world * wl.d * args.steps / elapsed
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(wl, world),
+        "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "traffic": traffic, "algorithmic_bytes_per_launch": local_bytes,
+                     "avg_launch_ms": avg_local_s * 1e3},
+        "global_step": {"bytes_per_launch": global_bytes, "avg_ms": avg_global_s * 1e3,
+                        "achieved_gbs": global_bytes / avg_global_s / 1e9,
+                        "frac": global_bytes / avg_global_s / 1e9 / peak,
+                        "note": "fused global step + statistics reduction, CUDA events around both"},
+        "optimizer_only_value": wl.d * args.steps / ((sum(local_ms) + sum(global_ms)) / 1e3),
+        "gpu_launches": args.steps * (2 * tau + 2),
+        "e2e": e2e,
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    print(json.dumps(line), flush=True)
+    run.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,244 @@
+/*
+ * dsm.h -- C ABI of the GB300 library for one global round of distributed
+ * sign momentum with local steps (arXiv 2411.17866, Algorithm 1).
+ *
+ * The problem (Sec. 1, Eq. (dist-opt)): n workers minimise the average of
+ * their local losses over a shared model x in R^d.  One global round
+ * (Algorithm 1) runs tau local base-optimizer steps on every worker's copy
+ * of the model, Eq. (local-steps), then averages the copies (the
+ * all-reduce), forms the sign-momentum update Eqs. (ut-update) and
+ * (model-update), updates the global momentum, Eq. (mom-update), and
+ * resets every worker copy to the new global model.
+ *
+ * Here the n workers are simulated as n replicas held in one GPU's memory;
+ * the all-reduce is an on-device reduction over the replicas.
+ *
+ * Memory and ownership
+ *   - The caller allocates one device buffer (the "arena", at least
+ *     dsm_state_bytes() bytes, 256-byte aligned) and keeps it alive until
+ *     dsm_destroy().  Every state of the method lives in it: global model x,
+ *     global momentum m, n worker replicas, n base-optimizer states, n
+ *     gradient buffers, the tile table and the statistics scratch.
+ *   - The library allocates no device memory.  It owns only the handle's
+ *     host-side metadata.
+ *   - Streams belong to the caller.  A stream argument is a cudaStream_t
+ *     passed as void*; NULL means the legacy default stream.
+ *
+ * Asynchrony
+ *   Every call that takes a stream only enqueues work on it, except where
+ *   its comment says it synchronises.  Calls on one handle must be issued in
+ *   the order of Algorithm 1 (the handle enforces it, see DSM_ESTATE).
+ *
+ * Errors
+ *   Every int-returning call returns DSM_OK (0) or a negative DSM_E* code
+ *   and never aborts the process; dsm_last_error() gives a message for the
+ *   calling thread's last failure.
+ *
+ * Thread safety: a handle is not thread-safe; distinct handles are
+ * independent.
+ */
+#ifndef DSM_H
+#define DSM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes ---------------------------------------------------- */
+#define DSM_OK      0
+#define DSM_EINVAL (-1)  /* bad argument (null pointer, n = 0, tau = 0, beta outside its range, ...) */
+#define DSM_ENOMEM (-2)  /* arena smaller than dsm_state_bytes() */
+#define DSM_EALIGN (-3)  /* arena not 256-byte aligned, or not device memory */
+#define DSM_ESTATE (-4)  /* call out of Algorithm 1's order (see dsm_local_step / dsm_global_step) */
+#define DSM_ECUDA  (-5)  /* a CUDA call or kernel launch failed; dsm_last_error() has its message */
+#define DSM_ERANGE (-6)  /* element range outside the model, worker index >= n, or a size beyond a limit */
+
+/* ---- enumerations ---------------------------------------------------- */
+/* Tensor kinds: only the initialisation depends on them (weights draw a
+ * hash value, LayerNorm weights start at 1, biases at 0). */
+#define DSM_KIND_WEIGHT 0
+#define DSM_KIND_BIAS   1
+#define DSM_KIND_LN_W   2
+#define DSM_KIND_LN_B   3
+
+/* Base optimizer of the local steps, Eq. (local-steps) (Appendix A). */
+#define DSM_BASE_ADAMW 0  /* Algorithm "AdamW" */
+#define DSM_BASE_SGDM  1  /* Algorithm "Polyak" (heavy ball); mu = 0 is plain SGD, Eq. (base-sgd) */
+
+/* Sign operator of the global step. */
+#define DSM_SIGN        0  /* deterministic sign, Eq. (model-update); sign(0) = 0 */
+#define DSM_RSIGN_ZERO  1  /* randomized sign, Eq. (rand-sign-2): sign(v) w.p. |v|/B, else 0 */
+#define DSM_RSIGN_PM    2  /* randomized sign, Eq. (rand-sign-1): sign(v) w.p. 1/2+|v|/(2B), else -sign(v) */
+
+/* Gradient storage type. */
+#define DSM_F32  0
+#define DSM_BF16 1
+
+/* Buffers for dsm_read_params / dsm_write_params. */
+#define DSM_BUF_X        0  /* global model x_{t,0} (fp32, d) */
+#define DSM_BUF_M        1  /* global momentum m_t (fp32, d) */
+#define DSM_BUF_REPLICA  2  /* worker replica x^{(i)} (fp32, d) */
+#define DSM_BUF_OPT_M    3  /* worker AdamW first moment, or SGD-momentum buffer (fp32, d) */
+#define DSM_BUF_OPT_V    4  /* worker AdamW second moment (fp32, d); AdamW only */
+#define DSM_BUF_GRAD     5  /* worker gradient buffer (fp32 or bf16 per grad_dtype, d) */
+
+typedef void* dsm_stream_t;  /* a cudaStream_t */
+
+/* One parameter tensor.  Tensors are packed in order into one flat model
+ * of d = sum(numel) elements; element e of the model is the "logical
+ * index" used by the synthetic generators and by dsm_read_params. */
+typedef struct {
+    uint64_t numel;       /* elements (0 allowed) */
+    float grad_scale;     /* s_T of the synthetic gradient generator */
+    uint32_t kind;        /* DSM_KIND_* */
+    uint32_t wd;          /* nonzero: decoupled weight decay applies (local and global) */
+    uint32_t reserved;    /* must be 0 */
+} dsm_tensor;
+
+typedef struct {
+    const dsm_tensor* tensors;  /* host array of count entries */
+    uint32_t count;
+} dsm_layout;
+
+/* Hyper-parameters.  Float fields are used as the fp32 values given. */
+typedef struct {
+    int32_t base;        /* DSM_BASE_* */
+    float lr;            /* gamma: local learning rate, also gamma_t of the global step; > 0 */
+    float b1, b2;        /* AdamW betas, in [0, 1) */
+    float eps;           /* AdamW epsilon, > 0 (the paper uses 1e-8) */
+    float wd;            /* AdamW decoupled weight decay, >= 0 */
+    float mu;            /* SGD-momentum coefficient, in [0, 1) */
+    float g_b1, g_b2;    /* global beta1, beta2 of Eqs. (ut-update), (mom-update), in [0, 1] */
+    float g_eta;         /* global learning rate eta of Eq. (model-update), >= 0 */
+    float g_wd;          /* global decoupled weight decay lambda, >= 0 */
+    int32_t sign_mode;   /* DSM_SIGN | DSM_RSIGN_ZERO | DSM_RSIGN_PM */
+    float rsign_B;       /* bound B of Eqs. (rand-sign-1/2); > 0 when randomized */
+    int32_t grad_dtype;  /* DSM_F32 | DSM_BF16 */
+    uint32_t reserved;   /* must be 0 */
+    uint64_t seed;       /* seed of the synthetic generators and of the Philox key */
+} dsm_hparams;
+
+/* Statistics of one global step for one tensor (Algorithm 1's quantities):
+ *   delta_sq  = sum_e Delta_e^2, Delta = (1/n) sum_i (x - x_i)      (pseudo-gradient norm, times gamma^2)
+ *   drift     = sum_e sum_i ((x_e - x_{i,e}) - Delta_e)^2           (spread of the workers around their mean)
+ *   zero_sign = #{e : applied sign = 0}
+ *   flips     = #{e : sign(u_e) != sign(Delta_e)}                    (momentum overrides the round's direction)
+ *   unanimous = #{e : sign(x_e - x_{i,e}) = sign(Delta_e) for every worker i}
+ *   clamped   = #{e : |u_e| > B} in the randomized modes, else 0
+ * Sums are accumulated in fp32 over the 8 elements of one thread and in
+ * fp64 beyond (relative error below 1e-5); counts are exact. */
+typedef struct {
+    double delta_sq;
+    double drift;
+    uint64_t zero_sign;
+    uint64_t flips;
+    uint64_t unanimous;
+    uint64_t clamped;
+} dsm_tensor_stats;
+
+/* Read-only description of a handle. */
+typedef struct {
+    uint64_t d;            /* model size */
+    uint64_t d_stride;     /* elements between consecutive workers in the replica/state/gradient buffers */
+    uint32_t n, tau;
+    uint32_t num_tensors, num_tiles;
+    uint64_t round;        /* t: completed global steps */
+    uint32_t local_steps;  /* k: local steps done in the current round (0..tau) */
+    float gamma;           /* gamma_t of the current round */
+} dsm_info;
+
+typedef struct dsm_handle dsm_handle;
+
+/* Bytes of device memory the arena must hold for this problem; 0 if the
+ * arguments are invalid (dsm_last_error() says why). */
+size_t dsm_state_bytes(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp);
+
+/* Create a handle over the caller's arena and initialise the state of
+ * Algorithm 1's first line: x_{0,0} from x0 (d fp32 values, host or device
+ * memory per x0_is_device) or, when x0 is NULL, from the hash
+ * initialisation (weights 0.02*(2u-1), LayerNorm weights 1, biases 0);
+ * m_0 = 0; every replica = x_{0,0}; base-optimizer states = 0.
+ * n in [1, 64], tau >= 1.  Enqueues the initialisation on stream and
+ * returns without waiting for it.  On failure *out is set to NULL. */
+int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hparams* hp,
+               void* dev_arena, size_t arena_bytes, const float* x0, int x0_is_device,
+               dsm_stream_t stream, dsm_handle** out);
+
+/* Set gamma_t for the current round: the local steps use it as their
+ * learning rate and the global step scales by it (Algorithm 1).  Only
+ * between rounds (no local step done yet in this round), else DSM_ESTATE;
+ * gamma must be > 0 and finite. */
+int dsm_set_gamma(dsm_handle* h, float gamma);
+
+/* Fill every worker's gradient buffer with the synthetic gradient of local
+ * step index `step` (conventionally t*tau + k):
+ *   g_i[e] = s_T*(u(seed,0,step,e) - 1/2) + fp32(0.1f*s_T)*(u(seed,1,i,e) - 1/2)
+ * with u the top 24 bits of a SplitMix64 output scaled by 2^-24, rounded to
+ * bf16 (nearest even) when grad_dtype is DSM_BF16.  Stands in for the
+ * backward pass.  Asynchronous. */
+int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream);
+
+/* Device pointer to worker `worker`'s gradient buffer (d elements of the
+ * gradient type; consecutive workers are d_stride elements apart), for a
+ * caller that writes gradients itself. */
+int dsm_grad_ptr(dsm_handle* h, uint32_t worker, void** dev_ptr);
+
+/* Copy all workers' gradients from src, a dense [n][d] array of the
+ * gradient type in host (src_is_device = 0; pinned memory makes it
+ * asynchronous) or device memory, into the gradient buffers. */
+int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream_t stream);
+
+/* Local step k of the current round on every worker, Eq. (local-steps):
+ * the base optimizer's update of each replica from its gradient buffer.
+ * AdamW's bias corrections use step count j = t*tau + k + 1 (the
+ * base-optimizer states persist across rounds; only the model is
+ * synchronised).  DSM_ESTATE if tau local steps were already done in this
+ * round.  Asynchronous. */
+int dsm_local_step(dsm_handle* h, dsm_stream_t stream);
+
+/* Global step of Algorithm 1 after the round's tau local steps (else
+ * DSM_ESTATE): Delta = (1/n) sum_{i=0..n-1} (x - x_i) (summed in worker
+ * order), u = b1 m + ((1-b1)/gamma) Delta, x' = x - eta gamma (S(u) + lambda x),
+ * m' = b2 m + ((1-b2)/gamma) Delta, every replica <- x', with S the sign
+ * or the randomized sign (Philox4x32-10, key (seed mod 2^32, t), counter
+ * floor(e/4), word e mod 4).  Also computes the per-tensor statistics.
+ * If stats is non-NULL (host memory, stats_count >= number of tensors) it
+ * copies them there and synchronises the stream; else it is asynchronous. */
+int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats, uint32_t stats_count);
+
+/* Device pointer to the per-tensor statistics of the last global step
+ * (num_tensors entries), valid once that step has run on the stream. */
+int dsm_stats_ptr(dsm_handle* h, const dsm_tensor_stats** dev_ptr);
+
+/* Copy elements [offset, offset+count) of buffer `which` (DSM_BUF_*) of
+ * worker `worker` (ignored for X and M) to dst (host or device memory).
+ * Elements are fp32 except DSM_BUF_GRAD, which has the gradient type.
+ * With a host dst the call synchronises the stream before returning. */
+int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64_t offset,
+                    uint64_t count, int dst_is_device, dsm_stream_t stream);
+
+/* The reverse of dsm_read_params (checkpoint restore, or a caller-set
+ * state).  With a host src the call synchronises the stream. */
+int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src, uint64_t offset,
+                     uint64_t count, int src_is_device, dsm_stream_t stream);
+
+/* Set the round counter t (checkpoint restore); only between rounds. */
+int dsm_set_round(dsm_handle* h, uint64_t round);
+
+int dsm_get_info(const dsm_handle* h, dsm_info* out);
+
+/* Release the handle's host metadata; the arena stays the caller's.
+ * NULL is accepted. */
+int dsm_destroy(dsm_handle* h);
+
+/* Message for the calling thread's last failed call ("" if none). */
+const char* dsm_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DSM_H */

@@ -1,0 +1,531 @@
+// Host side of the C ABI declared in include/dsm.h: argument checking, the
+// arena layout, the tile table, the per-launch scalars and the order of
+// Algorithm 1 (arXiv 2411.17866).  Allocates no device memory.
+
+#include "dsm.h"
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "dsm_internal.h"
+
+using namespace dsm;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(DSM_ECUDA, "%s: %s (%s)", what, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+constexpr uint64_t kAlign = 256;
+constexpr uint64_t kStrideAlign = 64;  // elements; keeps every worker slice 256-byte aligned
+constexpr uint64_t kMaxD = 1ull << 40;
+
+uint64_t round_up(uint64_t v, uint64_t a) { return (v + a - 1) / a * a; }
+
+// SplitMix64 (Steele, Lea, Flood, OOPSLA 2014) on the host: keys of the
+// synthetic generators.  key(seed, stream, idx) is output 1 + stream*2^40 + idx
+// of the generator seeded with `seed`.
+uint64_t sm64_finalise(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+uint64_t draw_key(uint64_t seed, uint64_t stream, uint64_t idx) {
+    const uint64_t j = 1ull + (stream << 40) + idx;
+    return sm64_finalise(seed + j * 0x9E3779B97F4A7C15ull);
+}
+
+bool finite(float v) { return std::isfinite(v); }
+
+// The arena: every region starts on a 256-byte boundary.
+struct ArenaLayout {
+    uint64_t d = 0, d_stride = 0;
+    uint32_t num_tensors = 0, num_tiles = 0;
+    uint64_t off_tensors = 0, off_tiles = 0, off_x = 0, off_m = 0, off_X = 0, off_om = 0, off_ov = 0,
+             off_grad = 0, off_partials = 0, off_stats = 0, total = 0;
+    size_t grad_esize = 4;
+};
+
+int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp, ArenaLayout* al) {
+    if (!layout || !hp) return fail(DSM_EINVAL, "layout and hparams must not be NULL");
+    if (layout->count == 0 || !layout->tensors) return fail(DSM_EINVAL, "layout has no tensors");
+    if (n == 0) return fail(DSM_EINVAL, "n (workers) must be >= 1");
+    if (n > kMaxWorkers) return fail(DSM_ERANGE, "n = %u exceeds the maximum of %u workers", n, kMaxWorkers);
+    if (hp->base != DSM_BASE_ADAMW && hp->base != DSM_BASE_SGDM)
+        return fail(DSM_EINVAL, "base optimizer %d unknown", hp->base);
+    if (!(finite(hp->lr) && hp->lr > 0.f)) return fail(DSM_EINVAL, "lr (gamma) must be finite and > 0");
+    if (hp->base == DSM_BASE_ADAMW) {
+        if (!(hp->b1 >= 0.f && hp->b1 < 1.f) || !(hp->b2 >= 0.f && hp->b2 < 1.f))
+            return fail(DSM_EINVAL, "AdamW betas must lie in [0, 1)");
+        if (!(finite(hp->eps) && hp->eps > 0.f)) return fail(DSM_EINVAL, "AdamW eps must be finite and > 0");
+        if (!(finite(hp->wd) && hp->wd >= 0.f)) return fail(DSM_EINVAL, "AdamW wd must be finite and >= 0");
+    } else {
+        if (!(hp->mu >= 0.f && hp->mu < 1.f)) return fail(DSM_EINVAL, "SGD momentum mu must lie in [0, 1)");
+    }
+    if (!(hp->g_b1 >= 0.f && hp->g_b1 <= 1.f) || !(hp->g_b2 >= 0.f && hp->g_b2 <= 1.f))
+        return fail(DSM_EINVAL, "global betas must lie in [0, 1]");
+    if (!(finite(hp->g_eta) && hp->g_eta >= 0.f)) return fail(DSM_EINVAL, "global eta must be finite and >= 0");
+    if (!(finite(hp->g_wd) && hp->g_wd >= 0.f)) return fail(DSM_EINVAL, "global lambda must be finite and >= 0");
+    if (hp->sign_mode != DSM_SIGN && hp->sign_mode != DSM_RSIGN_ZERO && hp->sign_mode != DSM_RSIGN_PM)
+        return fail(DSM_EINVAL, "sign mode %d unknown", hp->sign_mode);
+    if (hp->sign_mode != DSM_SIGN && !(finite(hp->rsign_B) && hp->rsign_B > 0.f))
+        return fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
+    if (hp->grad_dtype != DSM_F32 && hp->grad_dtype != DSM_BF16)
+        return fail(DSM_EINVAL, "gradient dtype %d unknown", hp->grad_dtype);
+    if (hp->reserved != 0) return fail(DSM_EINVAL, "hparams.reserved must be 0");
+
+    uint64_t d = 0, tiles = 0;
+    for (uint32_t i = 0; i < layout->count; ++i) {
+        const dsm_tensor& t = layout->tensors[i];
+        if (t.kind > DSM_KIND_LN_B) return fail(DSM_EINVAL, "tensor %u: kind %u unknown", i, t.kind);
+        if (!finite(t.grad_scale)) return fail(DSM_EINVAL, "tensor %u: grad_scale not finite", i);
+        if (t.reserved != 0) return fail(DSM_EINVAL, "tensor %u: reserved must be 0", i);
+        if (t.numel > kMaxD) return fail(DSM_ERANGE, "tensor %u: numel too large", i);
+        d += t.numel;
+        tiles += (t.numel + kTile - 1) / kTile;
+        if (d > kMaxD) return fail(DSM_ERANGE, "model larger than 2^40 elements");
+    }
+    if (d == 0) return fail(DSM_EINVAL, "the model has no elements (every tensor has numel 0)");
+    if (tiles * n >= (1ull << 32)) return fail(DSM_ERANGE, "too many tiles (%llu) for n = %u", (unsigned long long)tiles, n);
+
+    ArenaLayout a;
+    a.d = d;
+    a.d_stride = round_up(d, kStrideAlign);
+    a.num_tensors = layout->count;
+    a.num_tiles = static_cast<uint32_t>(tiles);
+    a.grad_esize = hp->grad_dtype == DSM_BF16 ? 2 : 4;
+    uint64_t off = 0;
+    auto take = [&](uint64_t bytes) {
+        const uint64_t o = off;
+        off = round_up(off + bytes, kAlign);
+        return o;
+    };
+    a.off_tensors = take(uint64_t(a.num_tensors) * sizeof(TensorDesc));
+    a.off_tiles = take(uint64_t(a.num_tiles) * sizeof(TileDesc));
+    a.off_x = take(a.d_stride * 4);
+    a.off_m = take(a.d_stride * 4);
+    a.off_X = take(uint64_t(n) * a.d_stride * 4);
+    a.off_om = take(uint64_t(n) * a.d_stride * 4);
+    a.off_ov = hp->base == DSM_BASE_ADAMW ? take(uint64_t(n) * a.d_stride * 4) : 0;
+    a.off_grad = take(uint64_t(n) * a.d_stride * a.grad_esize);
+    a.off_partials = take(uint64_t(a.num_tiles) * sizeof(StatPartial));
+    a.off_stats = take(uint64_t(a.num_tensors) * sizeof(TensorStats));
+    a.total = off;
+    *al = a;
+    return DSM_OK;
+}
+
+// Makes the handle's device current for the duration of a call.
+struct DeviceGuard {
+    int prev = -1;
+    cudaError_t err = cudaSuccess;
+    explicit DeviceGuard(int dev) {
+        err = cudaGetDevice(&prev);
+        if (err == cudaSuccess && prev != dev) err = cudaSetDevice(dev);
+        else if (err == cudaSuccess) prev = -1;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct dsm_handle {
+    int device = 0;
+    uint32_t n = 0, tau = 0;
+    dsm_hparams hp{};
+    ArenaLayout al;
+    char* arena = nullptr;
+    Problem prob{};
+    LaunchShape shape{};
+    std::vector<TensorDesc> tensors;
+    std::vector<TileDesc> tiles;
+    uint64_t t = 0;        // completed global steps
+    uint32_t k = 0;        // local steps done in this round
+    float gamma = 0.f;     // gamma_t of this round
+    double b1_pow = 1.0;   // beta1^j and beta2^j for the last local step count j
+    double b2_pow = 1.0;
+    uint64_t j = 0;        // local steps done since the start (AdamW step count)
+};
+
+namespace {
+
+cudaStream_t S(dsm_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
+
+float* buffer_ptr(dsm_handle* h, int which, uint32_t worker) {
+    const uint64_t ws = uint64_t(worker) * h->al.d_stride;
+    switch (which) {
+        case DSM_BUF_X: return h->prob.x;
+        case DSM_BUF_M: return h->prob.m;
+        case DSM_BUF_REPLICA: return h->prob.X + ws;
+        case DSM_BUF_OPT_M: return h->prob.opt_m + ws;
+        case DSM_BUF_OPT_V: return h->prob.opt_v ? h->prob.opt_v + ws : nullptr;
+        default: return nullptr;
+    }
+}
+
+// Resolves (which, worker) to a device address and element size.
+int resolve_buffer(dsm_handle* h, int which, uint32_t worker, uint64_t offset, uint64_t count, char** ptr,
+                   size_t* esize) {
+    if (which < DSM_BUF_X || which > DSM_BUF_GRAD) return fail(DSM_EINVAL, "buffer %d unknown", which);
+    const bool per_worker = which >= DSM_BUF_REPLICA;
+    if (per_worker && worker >= h->n) return fail(DSM_ERANGE, "worker %u >= n = %u", worker, h->n);
+    if (offset > h->al.d || count > h->al.d - offset)
+        return fail(DSM_ERANGE, "elements [%llu, %llu) outside the model of %llu", (unsigned long long)offset,
+                    (unsigned long long)(offset + count), (unsigned long long)h->al.d);
+    if (which == DSM_BUF_GRAD) {
+        *esize = h->al.grad_esize;
+        *ptr = static_cast<char*>(h->prob.grad) + (uint64_t(worker) * h->al.d_stride + offset) * *esize;
+        return DSM_OK;
+    }
+    float* b = buffer_ptr(h, which, per_worker ? worker : 0);
+    if (!b) return fail(DSM_EINVAL, "buffer %d does not exist for this base optimizer", which);
+    *esize = 4;
+    *ptr = reinterpret_cast<char*>(b + offset);
+    return DSM_OK;
+}
+
+int copy_kind(const void* host_or_dev, int is_device, bool to_device, cudaMemcpyKind* kind) {
+    (void)host_or_dev;
+    if (to_device) *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    else *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+    return DSM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t dsm_state_bytes(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp) {
+    ArenaLayout al;
+    if (check_layout_and_hp(layout, n, hp, &al) != DSM_OK) return 0;
+    return static_cast<size_t>(al.total);
+}
+
+int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hparams* hp, void* dev_arena,
+               size_t arena_bytes, const float* x0, int x0_is_device, dsm_stream_t stream, dsm_handle** out) {
+    if (!out) return fail(DSM_EINVAL, "out must not be NULL");
+    *out = nullptr;
+    ArenaLayout al;
+    int rc = check_layout_and_hp(layout, n, hp, &al);
+    if (rc != DSM_OK) return rc;
+    if (tau == 0) return fail(DSM_EINVAL, "tau (local steps per round) must be >= 1");
+    if (!dev_arena) return fail(DSM_EINVAL, "arena must not be NULL");
+    if (reinterpret_cast<uintptr_t>(dev_arena) % kAlign != 0)
+        return fail(DSM_EALIGN, "arena %p is not 256-byte aligned", dev_arena);
+    if (arena_bytes < al.total)
+        return fail(DSM_ENOMEM, "arena holds %zu bytes, the problem needs %llu", arena_bytes,
+                    (unsigned long long)al.total);
+
+    cudaPointerAttributes attr;
+    cudaError_t err = cudaPointerGetAttributes(&attr, dev_arena);
+    if (err != cudaSuccess) {
+        cudaGetLastError();
+        return cuda_fail(err, "cudaPointerGetAttributes(arena)");
+    }
+    if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
+        return fail(DSM_EALIGN, "arena %p is not device memory", dev_arena);
+
+    dsm_handle* h = new (std::nothrow) dsm_handle();
+    if (!h) return fail(DSM_ENOMEM, "out of host memory for the handle");
+    h->device = attr.device;
+    h->n = n;
+    h->tau = tau;
+    h->hp = *hp;
+    h->al = al;
+    h->arena = static_cast<char*>(dev_arena);
+    h->gamma = hp->lr;
+
+    // tensor and tile tables
+    h->tensors.resize(al.num_tensors);
+    h->tiles.reserve(al.num_tiles);
+    uint64_t off = 0;
+    for (uint32_t i = 0; i < al.num_tensors; ++i) {
+        const dsm_tensor& t = layout->tensors[i];
+        TensorDesc& td = h->tensors[i];
+        td.off = off;
+        td.numel = t.numel;
+        td.scale = t.grad_scale;
+        td.scale2 = 0.1f * t.grad_scale;
+        td.lam_local = t.wd ? hp->wd : 0.0f;
+        td.lam_global = t.wd ? hp->g_wd : 0.0f;
+        td.kind = t.kind;
+        td.tile_begin = static_cast<uint32_t>(h->tiles.size());
+        for (uint64_t o = 0; o < t.numel; o += kTile) {
+            TileDesc tl;
+            tl.start = off + o;
+            tl.len = static_cast<uint32_t>(t.numel - o < kTile ? t.numel - o : kTile);
+            tl.tensor = i;
+            h->tiles.push_back(tl);
+        }
+        td.tile_end = static_cast<uint32_t>(h->tiles.size());
+        td.pad = 0;
+        off += t.numel;
+    }
+
+    char* A = h->arena;
+    Problem& p = h->prob;
+    p.tensors = reinterpret_cast<const TensorDesc*>(A + al.off_tensors);
+    p.tiles = reinterpret_cast<const TileDesc*>(A + al.off_tiles);
+    p.num_tensors = al.num_tensors;
+    p.num_tiles = al.num_tiles;
+    p.n = n;
+    p.d_stride = al.d_stride;
+    p.x = reinterpret_cast<float*>(A + al.off_x);
+    p.m = reinterpret_cast<float*>(A + al.off_m);
+    p.X = reinterpret_cast<float*>(A + al.off_X);
+    p.opt_m = reinterpret_cast<float*>(A + al.off_om);
+    p.opt_v = hp->base == DSM_BASE_ADAMW ? reinterpret_cast<float*>(A + al.off_ov) : nullptr;
+    p.grad = A + al.off_grad;
+    p.grad_bf16 = hp->grad_dtype == DSM_BF16;
+    p.partials = reinterpret_cast<StatPartial*>(A + al.off_partials);
+    p.stats = reinterpret_cast<TensorStats*>(A + al.off_stats);
+
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) {
+        delete h;
+        return cuda_fail(guard.err, "cudaSetDevice");
+    }
+    cudaStream_t s = S(stream);
+    auto bail = [&](cudaError_t e, const char* what) {
+        delete h;
+        return cuda_fail(e, what);
+    };
+    if ((err = query_launch_shape(p, &h->shape)) != cudaSuccess) return bail(err, "occupancy query");
+    // The tables are copied from the handle's own vectors, which outlive the copies.
+    if ((err = cudaMemcpyAsync(A + al.off_tensors, h->tensors.data(), h->tensors.size() * sizeof(TensorDesc),
+                               cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return bail(err, "copy tensor table");
+    if ((err = cudaMemcpyAsync(A + al.off_tiles, h->tiles.data(), h->tiles.size() * sizeof(TileDesc),
+                               cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return bail(err, "copy tile table");
+    // m_0 = 0, base-optimizer states = 0, gradients = 0, statistics = 0
+    const uint64_t zero_from = al.off_m;
+    if ((err = cudaMemsetAsync(A + zero_from, 0, al.total - zero_from, s)) != cudaSuccess)
+        return bail(err, "zero the state");
+    if (x0) {
+        if ((err = cudaMemcpyAsync(p.x, x0, al.d * 4, x0_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice,
+                                   s)) != cudaSuccess)
+            return bail(err, "copy x0");
+    }
+    if ((err = launch_init(p, h->shape, draw_key(hp->seed, 2, 0), x0 ? 0 : 1, s)) != cudaSuccess)
+        return bail(err, "launch init");
+    *out = h;
+    return DSM_OK;
+}
+
+int dsm_set_gamma(dsm_handle* h, float gamma) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    if (!(finite(gamma) && gamma > 0.f)) return fail(DSM_EINVAL, "gamma must be finite and > 0");
+    if (h->k != 0) return fail(DSM_ESTATE, "gamma can change only between rounds (%u local steps done)", h->k);
+    h->gamma = gamma;
+    return DSM_OK;
+}
+
+int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    GradKeys k;
+    k.step = draw_key(h->hp.seed, 0, step);
+    for (uint32_t i = 0; i < kMaxWorkers; ++i) k.worker[i] = i < h->n ? draw_key(h->hp.seed, 1, i) : 0;
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaError_t err = launch_grad_fill(h->prob, h->shape, k, S(stream));
+    if (err != cudaSuccess) return cuda_fail(err, "launch grad fill");
+    return DSM_OK;
+}
+
+int dsm_grad_ptr(dsm_handle* h, uint32_t worker, void** dev_ptr) {
+    if (!h || !dev_ptr) return fail(DSM_EINVAL, "NULL argument");
+    if (worker >= h->n) return fail(DSM_ERANGE, "worker %u >= n = %u", worker, h->n);
+    *dev_ptr = static_cast<char*>(h->prob.grad) + uint64_t(worker) * h->al.d_stride * h->al.grad_esize;
+    return DSM_OK;
+}
+
+int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream_t stream) {
+    if (!h || !src) return fail(DSM_EINVAL, "NULL argument");
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    const size_t es = h->al.grad_esize;
+    cudaError_t err = cudaMemcpy2DAsync(h->prob.grad, h->al.d_stride * es, src, h->al.d * es, h->al.d * es, h->n,
+                                        src_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice,
+                                        S(stream));
+    if (err != cudaSuccess) return cuda_fail(err, "copy gradients");
+    return DSM_OK;
+}
+
+int dsm_local_step(dsm_handle* h, dsm_stream_t stream) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    if (h->k >= h->tau)
+        return fail(DSM_ESTATE, "all %u local steps of round %llu are done; call dsm_global_step", h->tau,
+                    (unsigned long long)h->t);
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaError_t err;
+    if (h->hp.base == DSM_BASE_ADAMW) {
+        // step count j = t*tau + k + 1; beta^j by successive float64 products
+        const double nb1 = h->b1_pow * double(h->hp.b1);
+        const double nb2 = h->b2_pow * double(h->hp.b2);
+        AdamScalars a;
+        a.b1 = h->hp.b1;
+        a.omb1 = float(1.0 - double(h->hp.b1));
+        a.b2 = h->hp.b2;
+        a.omb2 = float(1.0 - double(h->hp.b2));
+        a.bc1 = float(1.0 - nb1);
+        a.bc2 = float(1.0 - nb2);
+        a.lr = h->gamma;
+        a.eps = h->hp.eps;
+        err = launch_local_adamw(h->prob, h->shape, a, S(stream));
+        if (err != cudaSuccess) return cuda_fail(err, "launch AdamW local step");
+        h->b1_pow = nb1;
+        h->b2_pow = nb2;
+    } else {
+        SgdmScalars a;
+        a.mu = h->hp.mu;
+        a.lr = h->gamma;
+        err = launch_local_sgdm(h->prob, h->shape, a, S(stream));
+        if (err != cudaSuccess) return cuda_fail(err, "launch SGD-momentum local step");
+    }
+    h->j += 1;
+    h->k += 1;
+    return DSM_OK;
+}
+
+int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats, uint32_t stats_count) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    if (h->k != h->tau)
+        return fail(DSM_ESTATE, "global step needs %u local steps in this round, %u done", h->tau, h->k);
+    if (stats && stats_count < h->al.num_tensors)
+        return fail(DSM_EINVAL, "stats holds %u entries, the layout has %u tensors", stats_count, h->al.num_tensors);
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    GlobalScalars g;
+    g.b1 = h->hp.g_b1;
+    g.b2 = h->hp.g_b2;
+    g.c1 = float((1.0 - double(h->hp.g_b1)) / double(h->gamma));
+    g.c2 = float((1.0 - double(h->hp.g_b2)) / double(h->gamma));
+    g.eta_gamma = float(double(h->hp.g_eta) * double(h->gamma));
+    g.B = h->hp.rsign_B;
+    g.n_f = float(h->n);
+    g.sign_mode = h->hp.sign_mode;
+    g.philox_k0 = static_cast<uint32_t>(h->hp.seed & 0xFFFFFFFFull);
+    g.philox_k1 = static_cast<uint32_t>(h->t & 0xFFFFFFFFull);
+    cudaStream_t s = S(stream);
+    cudaError_t err = launch_global(h->prob, h->shape, g, s);
+    if (err != cudaSuccess) return cuda_fail(err, "launch global step");
+    err = launch_stats(h->prob, s);
+    if (err != cudaSuccess) return cuda_fail(err, "launch statistics");
+    h->t += 1;
+    h->k = 0;
+    if (stats) {
+        err = cudaMemcpyAsync(stats, h->prob.stats, size_t(h->al.num_tensors) * sizeof(TensorStats),
+                              cudaMemcpyDeviceToHost, s);
+        if (err != cudaSuccess) return cuda_fail(err, "copy statistics");
+        err = cudaStreamSynchronize(s);
+        if (err != cudaSuccess) return cuda_fail(err, "synchronise after the global step");
+    }
+    return DSM_OK;
+}
+
+int dsm_stats_ptr(dsm_handle* h, const dsm_tensor_stats** dev_ptr) {
+    if (!h || !dev_ptr) return fail(DSM_EINVAL, "NULL argument");
+    *dev_ptr = reinterpret_cast<const dsm_tensor_stats*>(h->prob.stats);
+    return DSM_OK;
+}
+
+int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64_t offset, uint64_t count,
+                    int dst_is_device, dsm_stream_t stream) {
+    if (!h || (!dst && count)) return fail(DSM_EINVAL, "NULL argument");
+    char* src;
+    size_t es;
+    int rc = resolve_buffer(h, which, worker, offset, count, &src, &es);
+    if (rc != DSM_OK) return rc;
+    if (count == 0) return DSM_OK;
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaMemcpyKind kind;
+    copy_kind(dst, dst_is_device, false, &kind);
+    cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
+    if (err != cudaSuccess) return cuda_fail(err, "read buffer");
+    if (!dst_is_device && (err = cudaStreamSynchronize(S(stream))) != cudaSuccess)
+        return cuda_fail(err, "synchronise after read");
+    return DSM_OK;
+}
+
+int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src, uint64_t offset, uint64_t count,
+                     int src_is_device, dsm_stream_t stream) {
+    if (!h || (!src && count)) return fail(DSM_EINVAL, "NULL argument");
+    char* dst;
+    size_t es;
+    int rc = resolve_buffer(h, which, worker, offset, count, &dst, &es);
+    if (rc != DSM_OK) return rc;
+    if (count == 0) return DSM_OK;
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaMemcpyKind kind;
+    copy_kind(src, src_is_device, true, &kind);
+    cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
+    if (err != cudaSuccess) return cuda_fail(err, "write buffer");
+    if (!src_is_device && (err = cudaStreamSynchronize(S(stream))) != cudaSuccess)
+        return cuda_fail(err, "synchronise after write");
+    return DSM_OK;
+}
+
+int dsm_set_round(dsm_handle* h, uint64_t round) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    if (h->k != 0) return fail(DSM_ESTATE, "the round counter can change only between rounds");
+    h->t = round;
+    h->j = round * h->tau;
+    double p1 = 1.0, p2 = 1.0;
+    for (uint64_t i = 0; i < h->j; ++i) {
+        p1 *= double(h->hp.b1);
+        p2 *= double(h->hp.b2);
+    }
+    h->b1_pow = p1;
+    h->b2_pow = p2;
+    return DSM_OK;
+}
+
+int dsm_get_info(const dsm_handle* h, dsm_info* out) {
+    if (!h || !out) return fail(DSM_EINVAL, "NULL argument");
+    out->d = h->al.d;
+    out->d_stride = h->al.d_stride;
+    out->n = h->n;
+    out->tau = h->tau;
+    out->num_tensors = h->al.num_tensors;
+    out->num_tiles = h->al.num_tiles;
+    out->round = h->t;
+    out->local_steps = h->k;
+    out->gamma = h->gamma;
+    return DSM_OK;
+}
+
+int dsm_destroy(dsm_handle* h) {
+    delete h;
+    return DSM_OK;
+}
+
+const char* dsm_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,123 @@
+// Internal interface between the C-ABI host code (dsm_api.cpp) and the
+// CUDA kernels (dsm_kernels.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace dsm {
+
+// Elements of one tile.  A tile lies inside one tensor; a tensor of numel
+// elements has ceil(numel / kTile) tiles.  One CTA of kThreads threads
+// processes one tile, kElemsPerThread consecutive elements per thread.
+constexpr uint32_t kThreads = 256;
+constexpr uint32_t kElemsPerThread = 8;
+constexpr uint32_t kTile = kThreads * kElemsPerThread;  // 2048
+constexpr uint32_t kMaxWorkers = 64;
+constexpr uint32_t kMaxUnrolledWorkers = 8;  // replicas held in registers by the global step
+
+// Per-tensor record in device memory (48 bytes).
+struct TensorDesc {
+    uint64_t off;          // first element in the packed model
+    uint64_t numel;
+    float scale;           // s_T
+    float scale2;          // fp32(0.1f * s_T)
+    float lam_local;       // AdamW decoupled weight decay for this tensor (0 if exempt)
+    float lam_global;      // global lambda for this tensor (0 if exempt)
+    uint32_t kind;
+    uint32_t tile_begin;   // tiles [tile_begin, tile_end) cover this tensor
+    uint32_t tile_end;
+    uint32_t pad;
+};
+static_assert(sizeof(TensorDesc) == 48, "TensorDesc layout");
+
+// Per-tile record in device memory (16 bytes).
+struct TileDesc {
+    uint64_t start;        // first element (logical index)
+    uint32_t len;          // 1..kTile
+    uint32_t tensor;
+};
+static_assert(sizeof(TileDesc) == 16, "TileDesc layout");
+
+// Per-tile partial statistics written by the global step (32 bytes).
+struct StatPartial {
+    double delta_sq;
+    double drift;
+    uint32_t zero_sign, flips, unanimous, clamped;
+};
+static_assert(sizeof(StatPartial) == 32, "StatPartial layout");
+
+// Per-tensor statistics (same layout as dsm_tensor_stats).
+struct TensorStats {
+    double delta_sq;
+    double drift;
+    unsigned long long zero_sign, flips, unanimous, clamped;
+};
+static_assert(sizeof(TensorStats) == 48, "TensorStats layout");
+
+// Views of the arena shared by the kernels.
+struct Problem {
+    const TensorDesc* tensors;
+    const TileDesc* tiles;
+    uint32_t num_tensors;
+    uint32_t num_tiles;
+    uint32_t n;
+    uint64_t d_stride;     // elements between workers
+    float* x;              // [d]
+    float* m;              // [d]
+    float* X;              // [n][d_stride] replicas
+    float* opt_m;          // [n][d_stride]
+    float* opt_v;          // [n][d_stride] (AdamW only)
+    void* grad;            // [n][d_stride], fp32 or bf16
+    int grad_bf16;
+    StatPartial* partials; // [num_tiles]
+    TensorStats* stats;    // [num_tensors]
+};
+
+// Scalars of one AdamW local step (all fp32, computed once on the host).
+struct AdamScalars {
+    float b1, omb1;        // beta1, 1 - beta1
+    float b2, omb2;        // beta2, 1 - beta2
+    float bc1, bc2;        // 1 - beta1^j, 1 - beta2^j
+    float lr, eps;
+};
+
+struct SgdmScalars {
+    float mu, lr;
+};
+
+struct GlobalScalars {
+    float b1, b2;          // global betas
+    float c1, c2;          // (1 - beta1)/gamma, (1 - beta2)/gamma
+    float eta_gamma;       // eta * gamma
+    float B;               // randomized-sign bound
+    float n_f;             // n as float (divisor of the average)
+    int sign_mode;
+    uint32_t philox_k0, philox_k1;
+};
+
+// SplitMix64 keys of one synthetic-gradient fill.
+struct GradKeys {
+    uint64_t step;                  // key(seed, 0, step)
+    uint64_t worker[kMaxWorkers];   // key(seed, 1, i)
+};
+
+// Launch shape: a persistent grid of `blocks` CTAs per kernel.
+struct LaunchShape {
+    int sms = 0;
+    int grid_grad = 0, grid_adamw = 0, grid_sgdm = 0, grid_global = 0, grid_init = 0;
+};
+
+// Launchers (dsm_kernels.cu).  Each returns the cudaError_t of its launch.
+cudaError_t query_launch_shape(const Problem& p, LaunchShape* out);
+cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t seed_key_init, int from_hash,
+                        cudaStream_t s);
+cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s);
+cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, cudaStream_t s);
+cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, cudaStream_t s);
+cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);
+cudaError_t launch_stats(const Problem& p, cudaStream_t s);
+
+}  // namespace dsm

@@ -1,0 +1,592 @@
+// CUDA kernels (sm_103a) for one global round of distributed sign momentum
+// with local steps (arXiv 2411.17866, Algorithm 1).
+//
+// Every kernel is a persistent, grid-stride loop over tiles of at most
+// kTile = 2048 elements that lie inside one tensor.  A CTA of 256 threads
+// takes one tile at a time; each thread owns 8 consecutive elements and
+// moves them with 16-byte loads and stores (two per fp32 stream, one per
+// bf16 stream).  The work is streaming and elementwise, so it is bound by
+// HBM bandwidth; nothing here is a contraction, and no tensor core is used.
+//
+// All method arithmetic uses the explicit round-to-nearest intrinsics
+// (__fadd_rn, __fmul_rn, __fdiv_rn, __fsqrt_rn, ...), which the compiler
+// never contracts into FMAs, so each result is the fp32 value of the
+// paper's expression evaluated one operation at a time.
+
+#include <cuda_bf16.h>
+
+#include "dsm_internal.h"
+
+namespace dsm {
+namespace {
+
+// ---------------------------------------------------------------------------
+// Counter-based generators
+// ---------------------------------------------------------------------------
+
+// SplitMix64 (Steele, Lea, Flood, OOPSLA 2014): output j of a generator
+// seeded with `state` is the state advanced j times by the golden-ratio
+// increment, passed through Stafford's variant-13 finaliser.
+constexpr uint64_t kGoldenGamma = 0x9E3779B97F4A7C15ull;
+
+__device__ __forceinline__ uint64_t sm64_finalise(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// u = top 24 bits of output e+1 of SplitMix64(key), times 2^-24 (exact in fp32).
+__device__ __forceinline__ float hash_uniform(uint64_t key, uint64_t e) {
+    const uint64_t h = sm64_finalise(key + (e + 1ull) * kGoldenGamma) >> 40;
+    return __fmul_rn(__uint2float_rn(static_cast<uint32_t>(h)), 5.9604644775390625e-08f);
+}
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC 2011): ten rounds of the
+// two-multiplier S-box with a Weyl key schedule.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        if (r) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    }
+    return c;
+}
+
+__device__ __forceinline__ uint4 philox_block(uint64_t q, uint32_t k0, uint32_t k1) {
+    return philox4x32_10(make_uint4(static_cast<uint32_t>(q), static_cast<uint32_t>(q >> 32), 0u, 0u), k0, k1);
+}
+
+__device__ __forceinline__ uint32_t word_of(const uint4& b, uint32_t i) {
+    return i == 0 ? b.x : (i == 1 ? b.y : (i == 2 ? b.z : b.w));
+}
+
+// r = (word >> 8) * 2^-24, exact in fp32.
+__device__ __forceinline__ float philox_unit(uint32_t w) {
+    return __fmul_rn(__uint2float_rn(w >> 8), 5.9604644775390625e-08f);
+}
+
+// ---------------------------------------------------------------------------
+// 16-byte streaming memory access
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+    const float4 a = __ldcs(reinterpret_cast<const float4*>(p));
+    const float4 b = __ldcs(reinterpret_cast<const float4*>(p) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+    __stcs(reinterpret_cast<float4*>(p), make_float4(v[0], v[1], v[2], v[3]));
+    __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(v[4], v[5], v[6], v[7]));
+}
+
+__device__ __forceinline__ void load8_bf16(const __nv_bfloat16* p, float (&v)[8]) {
+    const uint4 raw = __ldcs(reinterpret_cast<const uint4*>(p));
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // bf16 -> fp32 is exact: the bf16 bits are the top half
+        v[2 * i] = __uint_as_float(w[i] << 16);
+        v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+}
+
+__device__ __forceinline__ void store8_bf16(__nv_bfloat16* p, const float (&v)[8]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(v[2 * i]));
+        const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(v[2 * i + 1]));
+        w[i] = lo | (hi << 16);
+    }
+    __stcs(reinterpret_cast<uint4*>(p), make_uint4(w[0], w[1], w[2], w[3]));
+}
+
+__device__ __forceinline__ float load_grad1(const void* g, int bf16, uint64_t i) {
+    if (bf16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(g)[i]);
+    return reinterpret_cast<const float*>(g)[i];
+}
+
+// A thread's 8 elements take the vector path when the tile start is
+// 8-element aligned (so every stream is 16-byte aligned) and all 8 lie in
+// the tile; otherwise the thread handles its elements one at a time.
+__device__ __forceinline__ bool vector_ok(const TileDesc& td, uint32_t e0) {
+    return (td.start & 7u) == 0 && e0 + kElemsPerThread <= td.len;
+}
+
+// ---------------------------------------------------------------------------
+// Per-element arithmetic of the method
+// ---------------------------------------------------------------------------
+
+// Synthetic gradient: s*(u_step - 1/2) + s2*(u_worker - 1/2), left to right.
+__device__ __forceinline__ float step_term(float s, float u) { return __fmul_rn(s, __fsub_rn(u, 0.5f)); }
+__device__ __forceinline__ float grad_value(float a, float s2, float u2) {
+    return __fadd_rn(a, __fmul_rn(s2, __fsub_rn(u2, 0.5f)));
+}
+
+// AdamW (Appendix A): m <- b1 m + (1-b1) g; v <- b2 v + (1-b2) g*g;
+// x <- x - lr (mhat/(sqrt(vhat)+eps) + lam x), mhat = m/bc1, vhat = v/bc2.
+__device__ __forceinline__ void adamw_elem(float& x, float& m, float& v, float g, const AdamScalars& a, float lam) {
+    m = __fadd_rn(__fmul_rn(a.b1, m), __fmul_rn(a.omb1, g));
+    v = __fadd_rn(__fmul_rn(a.b2, v), __fmul_rn(a.omb2, __fmul_rn(g, g)));
+    const float mhat = __fdiv_rn(m, a.bc1);
+    const float vhat = __fdiv_rn(v, a.bc2);
+    const float den = __fadd_rn(__fsqrt_rn(vhat), a.eps);
+    const float upd = __fadd_rn(__fdiv_rn(mhat, den), __fmul_rn(lam, x));
+    x = __fsub_rn(x, __fmul_rn(a.lr, upd));
+}
+
+// Polyak momentum (Appendix A): buf <- mu buf + g; x <- x - lr buf.
+__device__ __forceinline__ void sgdm_elem(float& x, float& b, float g, const SgdmScalars& a) {
+    b = __fadd_rn(__fmul_rn(a.mu, b), g);
+    x = __fsub_rn(x, __fmul_rn(a.lr, b));
+}
+
+__device__ __forceinline__ int sgn(float v) { return (v > 0.f) - (v < 0.f); }
+
+// Applied sign S(u): deterministic sign, or the randomized sign of
+// Eq. (rand-sign-2) (mode 1) / Eq. (rand-sign-1) (mode 2) with uniform r.
+__device__ __forceinline__ float applied_sign(float u, const GlobalScalars& g, float r) {
+    const float s = static_cast<float>(sgn(u));
+    if (g.sign_mode == 0) return s;
+    const float p = fminf(__fdiv_rn(fabsf(u), g.B), 1.0f);
+    if (g.sign_mode == 1) return r < p ? s : 0.0f;
+    const float q = __fadd_rn(0.5f, __fmul_rn(0.5f, p));
+    return r < q ? s : -s;
+}
+
+struct ThreadStats {
+    float dsq = 0.f, drift = 0.f;
+    uint32_t zero = 0, flips = 0, unanimous = 0, clamped = 0;
+};
+
+// Global step on one element given x, m and the worker differences d_i = x - x_i:
+// Delta = (sum_i d_i)/n; u = b1 m + c1 Delta; x' = x - eta*gamma (S(u) + lam x);
+// m' = b2 m + c2 Delta.  Accumulates the statistics of the element.
+template <int NW>
+__device__ __forceinline__ void global_elem(float& x, float& m, const float (&dif)[NW], int nw,
+                                            const GlobalScalars& g, float lam, float r, ThreadStats& st) {
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < NW; ++i)
+        if (i < nw) acc = __fadd_rn(acc, dif[i]);
+    const float D = __fdiv_rn(acc, g.n_f);
+    const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
+    const float s = applied_sign(u, g, r);
+    const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
+    const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    // statistics
+    const int sD = sgn(D);
+    st.dsq = __fadd_rn(st.dsq, __fmul_rn(D, D));
+    bool unan = true;
+    float dr = 0.f;
+#pragma unroll
+    for (int i = 0; i < NW; ++i) {
+        if (i < nw) {
+            const float e = __fsub_rn(dif[i], D);
+            dr = __fadd_rn(dr, __fmul_rn(e, e));
+            unan = unan && (sgn(dif[i]) == sD);
+        }
+    }
+    st.drift = __fadd_rn(st.drift, dr);
+    st.zero += (s == 0.f);
+    st.flips += (sgn(u) != sD);
+    st.unanimous += unan;
+    st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
+    x = xn;
+    m = mn;
+}
+
+// Fixed-order CTA reduction of the per-thread statistics into one partial.
+__device__ __forceinline__ void reduce_stats(const ThreadStats& st, StatPartial* out) {
+    __shared__ double s_d[kThreads / 32][2];
+    __shared__ uint32_t s_c[kThreads / 32][4];
+    double a = static_cast<double>(st.dsq), b = static_cast<double>(st.drift);
+    uint32_t c0 = st.zero, c1 = st.flips, c2 = st.unanimous, c3 = st.clamped;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        a += __shfl_down_sync(0xffffffffu, a, off);
+        b += __shfl_down_sync(0xffffffffu, b, off);
+        c0 += __shfl_down_sync(0xffffffffu, c0, off);
+        c1 += __shfl_down_sync(0xffffffffu, c1, off);
+        c2 += __shfl_down_sync(0xffffffffu, c2, off);
+        c3 += __shfl_down_sync(0xffffffffu, c3, off);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        s_d[warp][0] = a; s_d[warp][1] = b;
+        s_c[warp][0] = c0; s_c[warp][1] = c1; s_c[warp][2] = c2; s_c[warp][3] = c3;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        constexpr int kWarps = kThreads / 32;
+        a = lane < kWarps ? s_d[lane][0] : 0.0;
+        b = lane < kWarps ? s_d[lane][1] : 0.0;
+        c0 = lane < kWarps ? s_c[lane][0] : 0u;
+        c1 = lane < kWarps ? s_c[lane][1] : 0u;
+        c2 = lane < kWarps ? s_c[lane][2] : 0u;
+        c3 = lane < kWarps ? s_c[lane][3] : 0u;
+#pragma unroll
+        for (int off = kWarps / 2; off > 0; off >>= 1) {
+            a += __shfl_down_sync(0xffffffffu, a, off);
+            b += __shfl_down_sync(0xffffffffu, b, off);
+            c0 += __shfl_down_sync(0xffffffffu, c0, off);
+            c1 += __shfl_down_sync(0xffffffffu, c1, off);
+            c2 += __shfl_down_sync(0xffffffffu, c2, off);
+            c3 += __shfl_down_sync(0xffffffffu, c3, off);
+        }
+        if (lane == 0) {
+            StatPartial p;
+            p.delta_sq = a; p.drift = b;
+            p.zero_sign = c0; p.flips = c1; p.unanimous = c2; p.clamped = c3;
+            *out = p;
+        }
+    }
+    __syncthreads();  // the shared arrays are reused by the next tile
+}
+
+// ---------------------------------------------------------------------------
+// Kernels
+// ---------------------------------------------------------------------------
+
+// Initial state: x (hash init by tensor kind, or as already copied) and every replica = x.
+__global__ void __launch_bounds__(kThreads) k_init(Problem p, uint64_t key_init, int from_hash) {
+    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = p.tiles[ti];
+        const uint32_t kind = p.tensors[td.tensor].kind;
+        const uint32_t e0 = threadIdx.x * kElemsPerThread;
+        const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+        for (uint32_t e = e0; e < e1; ++e) {
+            const uint64_t gi = td.start + e;
+            float v;
+            if (from_hash) {
+                if (kind == 0) {
+                    const float u = hash_uniform(key_init, gi);
+                    v = __fmul_rn(0.02f, __fsub_rn(__fmul_rn(2.0f, u), 1.0f));
+                } else {
+                    v = (kind == 2) ? 1.0f : 0.0f;
+                }
+                p.x[gi] = v;
+            } else {
+                v = p.x[gi];
+            }
+            for (uint32_t w = 0; w < p.n; ++w) p.X[w * p.d_stride + gi] = v;
+        }
+    }
+}
+
+// K1: synthetic gradients of one local step for every worker.
+template <bool kBf16>
+__global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
+    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = p.tiles[ti];
+        const TensorDesc& T = p.tensors[td.tensor];
+        const float s = T.scale, s2 = T.scale2;
+        const uint32_t e0 = threadIdx.x * kElemsPerThread;
+        if (vector_ok(td, e0)) {
+            const uint64_t gi = td.start + e0;
+            float a[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) a[j] = step_term(s, hash_uniform(k.step, gi + j));
+            for (uint32_t w = 0; w < p.n; ++w) {
+                float g[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) g[j] = grad_value(a[j], s2, hash_uniform(k.worker[w], gi + j));
+                const uint64_t o = w * p.d_stride + gi;
+                if (kBf16) store8_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
+                else store8(reinterpret_cast<float*>(p.grad) + o, g);
+            }
+        } else {
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t gi = td.start + e;
+                const float a = step_term(s, hash_uniform(k.step, gi));
+                for (uint32_t w = 0; w < p.n; ++w) {
+                    const float g = grad_value(a, s2, hash_uniform(k.worker[w], gi));
+                    const uint64_t o = w * p.d_stride + gi;
+                    if (kBf16) reinterpret_cast<__nv_bfloat16*>(p.grad)[o] = __float2bfloat16_rn(g);
+                    else reinterpret_cast<float*>(p.grad)[o] = g;
+                }
+            }
+        }
+    }
+}
+
+// K2: one AdamW local step on every worker (work item = (worker, tile)).
+template <bool kBf16>
+__global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars a) {
+    const uint32_t items = p.num_tiles * p.n;
+    for (uint32_t item = blockIdx.x; item < items; item += gridDim.x) {
+        const uint32_t w = item / p.num_tiles;
+        const uint32_t ti = item - w * p.num_tiles;
+        const TileDesc td = p.tiles[ti];
+        const float lam = p.tensors[td.tensor].lam_local;
+        const uint64_t base = w * p.d_stride + td.start;
+        const uint32_t e0 = threadIdx.x * kElemsPerThread;
+        if (vector_ok(td, e0)) {
+            float x[8], m[8], v[8], g[8];
+            load8(p.X + base + e0, x);
+            load8(p.opt_m + base + e0, m);
+            load8(p.opt_v + base + e0, v);
+            if (kBf16) load8_bf16(reinterpret_cast<const __nv_bfloat16*>(p.grad) + base + e0, g);
+            else load8(reinterpret_cast<const float*>(p.grad) + base + e0, g);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) adamw_elem(x[j], m[j], v[j], g[j], a, lam);
+            store8(p.X + base + e0, x);
+            store8(p.opt_m + base + e0, m);
+            store8(p.opt_v + base + e0, v);
+        } else {
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t i = base + e;
+                float x = p.X[i], m = p.opt_m[i], v = p.opt_v[i];
+                adamw_elem(x, m, v, load_grad1(p.grad, kBf16, i), a, lam);
+                p.X[i] = x; p.opt_m[i] = m; p.opt_v[i] = v;
+            }
+        }
+    }
+}
+
+// K3: one SGD-momentum local step on every worker.
+template <bool kBf16>
+__global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars a) {
+    const uint32_t items = p.num_tiles * p.n;
+    for (uint32_t item = blockIdx.x; item < items; item += gridDim.x) {
+        const uint32_t w = item / p.num_tiles;
+        const uint32_t ti = item - w * p.num_tiles;
+        const TileDesc td = p.tiles[ti];
+        const uint64_t base = w * p.d_stride + td.start;
+        const uint32_t e0 = threadIdx.x * kElemsPerThread;
+        if (vector_ok(td, e0)) {
+            float x[8], b[8], g[8];
+            load8(p.X + base + e0, x);
+            load8(p.opt_m + base + e0, b);
+            if (kBf16) load8_bf16(reinterpret_cast<const __nv_bfloat16*>(p.grad) + base + e0, g);
+            else load8(reinterpret_cast<const float*>(p.grad) + base + e0, g);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sgdm_elem(x[j], b[j], g[j], a);
+            store8(p.X + base + e0, x);
+            store8(p.opt_m + base + e0, b);
+        } else {
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t i = base + e;
+                float x = p.X[i], b = p.opt_m[i];
+                sgdm_elem(x, b, load_grad1(p.grad, kBf16, i), a);
+                p.X[i] = x; p.opt_m[i] = b;
+            }
+        }
+    }
+}
+
+// K4: the fused global step (average over the replicas, sign-momentum update,
+// momentum update, reset of every replica) with per-tile statistics.
+// NW > 0: exactly NW replicas, held in registers.  NW == 0: any n, one
+// element at a time, reading each replica twice.
+template <int NW>
+__global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g) {
+    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = p.tiles[ti];
+        const float lam = p.tensors[td.tensor].lam_global;
+        const uint32_t e0 = threadIdx.x * kElemsPerThread;
+        ThreadStats st;
+        if (NW > 0 && vector_ok(td, e0)) {
+            constexpr int W = NW > 0 ? NW : 1;
+            const uint64_t gi = td.start + e0;
+            float x[8], m[8], r[W][8];
+            load8(p.x + gi, x);
+            load8(p.m + gi, m);
+#pragma unroll
+            for (int i = 0; i < W; ++i) load8(p.X + i * p.d_stride + gi, r[i]);
+            float ru[8];
+            if (g.sign_mode != 0) {  // elements gi..gi+7 are the words of two Philox blocks
+                const uint4 b0 = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                const uint4 b1 = philox_block((gi >> 2) + 1, g.philox_k0, g.philox_k1);
+                ru[0] = philox_unit(b0.x); ru[1] = philox_unit(b0.y); ru[2] = philox_unit(b0.z); ru[3] = philox_unit(b0.w);
+                ru[4] = philox_unit(b1.x); ru[5] = philox_unit(b1.y); ru[6] = philox_unit(b1.z); ru[7] = philox_unit(b1.w);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) ru[j] = 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                float dif[W];
+#pragma unroll
+                for (int i = 0; i < W; ++i) dif[i] = __fsub_rn(x[j], r[i][j]);
+                global_elem<W>(x[j], m[j], dif, W, g, lam, ru[j], st);
+            }
+            store8(p.x + gi, x);
+            store8(p.m + gi, m);
+#pragma unroll
+            for (int i = 0; i < W; ++i) store8(p.X + i * p.d_stride + gi, x);
+        } else {
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t gi = td.start + e;
+                float x = p.x[gi], m = p.m[gi];
+                float r = 0.f;
+                if (g.sign_mode != 0)
+                    r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
+                // one element, any number of workers: the worker differences are read
+                // once for the average and once more for the statistics
+                float acc = 0.f;
+                for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x, p.X[i * p.d_stride + gi]));
+                const float D = __fdiv_rn(acc, g.n_f);
+                const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
+                const float s = applied_sign(u, g, r);
+                const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
+                const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+                const int sD = sgn(D);
+                float dr = 0.f;
+                bool unan = true;
+                for (uint32_t i = 0; i < p.n; ++i) {
+                    const float di = __fsub_rn(x, p.X[i * p.d_stride + gi]);
+                    const float ei = __fsub_rn(di, D);
+                    dr = __fadd_rn(dr, __fmul_rn(ei, ei));
+                    unan = unan && (sgn(di) == sD);
+                }
+                st.dsq = __fadd_rn(st.dsq, __fmul_rn(D, D));
+                st.drift = __fadd_rn(st.drift, dr);
+                st.zero += (s == 0.f);
+                st.flips += (sgn(u) != sD);
+                st.unanimous += unan;
+                st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
+                p.x[gi] = xn;
+                p.m[gi] = mn;
+                for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = xn;
+            }
+        }
+        reduce_stats(st, p.partials + ti);
+    }
+}
+
+// K5: per-tensor statistics from the tile partials, in a fixed order.
+__global__ void __launch_bounds__(kThreads) k_stats(Problem p) {
+    const uint32_t T = blockIdx.x;
+    const TensorDesc td = p.tensors[T];
+    double a = 0.0, b = 0.0;
+    unsigned long long c0 = 0, c1 = 0, c2 = 0, c3 = 0;
+    for (uint32_t t = td.tile_begin + threadIdx.x; t < td.tile_end; t += blockDim.x) {
+        const StatPartial q = p.partials[t];
+        a += q.delta_sq; b += q.drift;
+        c0 += q.zero_sign; c1 += q.flips; c2 += q.unanimous; c3 += q.clamped;
+    }
+    __shared__ double s_d[kThreads][2];
+    __shared__ unsigned long long s_c[kThreads][4];
+    s_d[threadIdx.x][0] = a; s_d[threadIdx.x][1] = b;
+    s_c[threadIdx.x][0] = c0; s_c[threadIdx.x][1] = c1; s_c[threadIdx.x][2] = c2; s_c[threadIdx.x][3] = c3;
+    __syncthreads();
+    for (uint32_t off = kThreads / 2; off > 0; off >>= 1) {
+        if (threadIdx.x < off) {
+            s_d[threadIdx.x][0] += s_d[threadIdx.x + off][0];
+            s_d[threadIdx.x][1] += s_d[threadIdx.x + off][1];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) s_c[threadIdx.x][k] += s_c[threadIdx.x + off][k];
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        TensorStats o;
+        o.delta_sq = s_d[0][0]; o.drift = s_d[0][1];
+        o.zero_sign = s_c[0][0]; o.flips = s_c[0][1]; o.unanimous = s_c[0][2]; o.clamped = s_c[0][3];
+        p.stats[T] = o;
+    }
+}
+
+template <typename K>
+int grid_for(K kernel, int sms) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, 0) != cudaSuccess || per_sm < 1)
+        per_sm = 1;
+    return sms * per_sm;
+}
+
+using GlobalKernel = void (*)(Problem, GlobalScalars);
+
+GlobalKernel global_kernel_for(uint32_t n) {
+    switch (n) {
+        case 1: return k_global<1>;
+        case 2: return k_global<2>;
+        case 3: return k_global<3>;
+        case 4: return k_global<4>;
+        case 5: return k_global<5>;
+        case 6: return k_global<6>;
+        case 7: return k_global<7>;
+        case 8: return k_global<8>;
+        default: return k_global<0>;
+    }
+}
+
+}  // namespace
+
+cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    out->sms = sms;
+    out->grid_init = grid_for(k_init, sms);
+    out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms) : grid_for(k_grad_fill<false>, sms);
+    out->grid_adamw = p.grad_bf16 ? grid_for(k_local_adamw<true>, sms) : grid_for(k_local_adamw<false>, sms);
+    out->grid_sgdm = p.grad_bf16 ? grid_for(k_local_sgdm<true>, sms) : grid_for(k_local_sgdm<false>, sms);
+    out->grid_global = grid_for(global_kernel_for(p.n), sms);
+    return cudaGetLastError();
+}
+
+static int clamp_grid(int grid, uint64_t items) {
+    if (items == 0) return 0;
+    return static_cast<int>(items < static_cast<uint64_t>(grid) ? items : static_cast<uint64_t>(grid));
+}
+
+cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t key_init, int from_hash, cudaStream_t s) {
+    const int grid = clamp_grid(ls.grid_init, p.num_tiles);
+    if (grid == 0) return cudaSuccess;
+    k_init<<<grid, kThreads, 0, s>>>(p, key_init, from_hash);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s) {
+    const int grid = clamp_grid(ls.grid_grad, p.num_tiles);
+    if (grid == 0) return cudaSuccess;
+    if (p.grad_bf16) k_grad_fill<true><<<grid, kThreads, 0, s>>>(p, k);
+    else k_grad_fill<false><<<grid, kThreads, 0, s>>>(p, k);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, cudaStream_t s) {
+    const int grid = clamp_grid(ls.grid_adamw, static_cast<uint64_t>(p.num_tiles) * p.n);
+    if (grid == 0) return cudaSuccess;
+    if (p.grad_bf16) k_local_adamw<true><<<grid, kThreads, 0, s>>>(p, a);
+    else k_local_adamw<false><<<grid, kThreads, 0, s>>>(p, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, cudaStream_t s) {
+    const int grid = clamp_grid(ls.grid_sgdm, static_cast<uint64_t>(p.num_tiles) * p.n);
+    if (grid == 0) return cudaSuccess;
+    if (p.grad_bf16) k_local_sgdm<true><<<grid, kThreads, 0, s>>>(p, a);
+    else k_local_sgdm<false><<<grid, kThreads, 0, s>>>(p, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s) {
+    const int grid = clamp_grid(ls.grid_global, p.num_tiles);
+    if (grid == 0) return cudaSuccess;
+    global_kernel_for(p.n)<<<grid, kThreads, 0, s>>>(p, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stats(const Problem& p, cudaStream_t s) {
+    if (p.num_tensors == 0) return cudaSuccess;
+    k_stats<<<p.num_tensors, kThreads, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace dsm

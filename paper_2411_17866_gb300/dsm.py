@@ -1,0 +1,325 @@
+"""Python binding of libdsm.so (include/dsm.h): argument marshalling only.
+
+Each ``dsm_*`` function here calls the C function of the same name through
+ctypes and raises :class:`DsmError` on a negative return code.  Every step
+of the method runs in the library's CUDA kernels; PyTorch only supplies the
+device memory (the arena, a uint8 tensor) and the current CUDA stream.
+
+:class:`DistributedSignMomentum` is a thin convenience wrapper that owns the
+arena tensor and a handle and exposes the round as Python methods.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, byref, c_char_p, c_float, c_int, c_int32, c_size_t, c_uint32, c_uint64, c_void_p
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdsm.so")
+
+DSM_OK, DSM_EINVAL, DSM_ENOMEM, DSM_EALIGN, DSM_ESTATE, DSM_ECUDA, DSM_ERANGE = 0, -1, -2, -3, -4, -5, -6
+KIND_WEIGHT, KIND_BIAS, KIND_LN_W, KIND_LN_B = 0, 1, 2, 3
+BASE_ADAMW, BASE_SGDM = 0, 1
+SIGN, RSIGN_ZERO, RSIGN_PM = 0, 1, 2
+F32, BF16 = 0, 1
+BUF_X, BUF_M, BUF_REPLICA, BUF_OPT_M, BUF_OPT_V, BUF_GRAD = 0, 1, 2, 3, 4, 5
+
+ERROR_NAMES = {DSM_EINVAL: "DSM_EINVAL", DSM_ENOMEM: "DSM_ENOMEM", DSM_EALIGN: "DSM_EALIGN",
+               DSM_ESTATE: "DSM_ESTATE", DSM_ECUDA: "DSM_ECUDA", DSM_ERANGE: "DSM_ERANGE"}
+
+
+class DsmError(RuntimeError):
+    def __init__(self, code: int, func: str, msg: str):
+        super().__init__(f"{func} failed with {ERROR_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class dsm_tensor(ctypes.Structure):
+    _fields_ = [("numel", c_uint64), ("grad_scale", c_float), ("kind", c_uint32), ("wd", c_uint32),
+                ("reserved", c_uint32)]
+
+
+class dsm_layout(ctypes.Structure):
+    _fields_ = [("tensors", POINTER(dsm_tensor)), ("count", c_uint32)]
+
+
+class dsm_hparams(ctypes.Structure):
+    _fields_ = [("base", c_int32), ("lr", c_float), ("b1", c_float), ("b2", c_float), ("eps", c_float),
+                ("wd", c_float), ("mu", c_float), ("g_b1", c_float), ("g_b2", c_float), ("g_eta", c_float),
+                ("g_wd", c_float), ("sign_mode", c_int32), ("rsign_B", c_float), ("grad_dtype", c_int32),
+                ("reserved", c_uint32), ("seed", c_uint64)]
+
+
+class dsm_tensor_stats(ctypes.Structure):
+    _fields_ = [("delta_sq", ctypes.c_double), ("drift", ctypes.c_double), ("zero_sign", c_uint64),
+                ("flips", c_uint64), ("unanimous", c_uint64), ("clamped", c_uint64)]
+
+    def as_dict(self):
+        return {f: getattr(self, f) for f, _ in self._fields_}
+
+
+class dsm_info(ctypes.Structure):
+    _fields_ = [("d", c_uint64), ("d_stride", c_uint64), ("n", c_uint32), ("tau", c_uint32),
+                ("num_tensors", c_uint32), ("num_tiles", c_uint32), ("round", c_uint64),
+                ("local_steps", c_uint32), ("gamma", c_float)]
+
+
+_PROTOS = {
+    "dsm_state_bytes": (c_size_t, [POINTER(dsm_layout), c_uint32, POINTER(dsm_hparams)]),
+    "dsm_create": (c_int, [POINTER(dsm_layout), c_uint32, c_uint32, POINTER(dsm_hparams), c_void_p, c_size_t,
+                           c_void_p, c_int, c_void_p, POINTER(c_void_p)]),
+    "dsm_set_gamma": (c_int, [c_void_p, c_float]),
+    "dsm_fill_synthetic_grads": (c_int, [c_void_p, c_uint64, c_void_p]),
+    "dsm_grad_ptr": (c_int, [c_void_p, c_uint32, POINTER(c_void_p)]),
+    "dsm_load_grads": (c_int, [c_void_p, c_void_p, c_int, c_void_p]),
+    "dsm_local_step": (c_int, [c_void_p, c_void_p]),
+    "dsm_global_step": (c_int, [c_void_p, c_void_p, POINTER(dsm_tensor_stats), c_uint32]),
+    "dsm_stats_ptr": (c_int, [c_void_p, POINTER(c_void_p)]),
+    "dsm_read_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
+    "dsm_write_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
+    "dsm_set_round": (c_int, [c_void_p, c_uint64]),
+    "dsm_get_info": (c_int, [c_void_p, POINTER(dsm_info)]),
+    "dsm_destroy": (c_int, [c_void_p]),
+    "dsm_last_error": (c_char_p, []),
+}
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libdsm.so; raises if it has not been built (there is no fallback)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'` "
+                           "(the CUDA library is required; there is no CPU fallback)")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in _PROTOS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def last_error() -> str:
+    return load_library().dsm_last_error().decode()
+
+
+def _check(rc: int, func: str) -> None:
+    if rc != DSM_OK:
+        raise DsmError(rc, func, last_error())
+
+
+def _stream(stream) -> c_void_p:
+    """A cudaStream_t from a torch stream, an int handle, or None (torch's current stream)."""
+    if stream is None:
+        import torch
+        return c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return c_void_p(stream)
+    return c_void_p(stream.cuda_stream)
+
+
+def make_layout(tensors):
+    """A dsm_layout from objects with numel, grad_scale, kind and wd; keep the result alive while used."""
+    arr = (dsm_tensor * len(tensors))()
+    for i, t in enumerate(tensors):
+        arr[i].numel = int(t.numel)
+        arr[i].grad_scale = float(t.grad_scale)
+        arr[i].kind = int(t.kind)
+        arr[i].wd = int(getattr(t, "wd", 1))
+        arr[i].reserved = 0
+    lay = dsm_layout(ctypes.cast(arr, POINTER(dsm_tensor)), len(tensors))
+    lay._keep = arr
+    return lay
+
+
+def make_hparams(hp) -> dsm_hparams:
+    """A dsm_hparams from an object with the same field names."""
+    h = dsm_hparams()
+    for name, _ in dsm_hparams._fields_:
+        if name == "reserved":
+            continue
+        setattr(h, name, getattr(hp, name))
+    h.reserved = 0
+    return h
+
+
+# ---- the C functions, same names ----------------------------------------
+
+def dsm_state_bytes(layout: dsm_layout, n: int, hp: dsm_hparams) -> int:
+    nb = load_library().dsm_state_bytes(byref(layout), n, byref(hp))
+    if nb == 0:
+        raise DsmError(DSM_EINVAL, "dsm_state_bytes", last_error())
+    return nb
+
+
+def dsm_create(layout, n, tau, hp, arena_ptr: int, arena_bytes: int, x0_ptr=None, x0_is_device=False,
+               stream=None) -> c_void_p:
+    h = c_void_p()
+    rc = load_library().dsm_create(byref(layout), n, tau, byref(hp), c_void_p(arena_ptr), arena_bytes,
+                                   c_void_p(x0_ptr) if x0_ptr else None, int(bool(x0_is_device)),
+                                   _stream(stream), byref(h))
+    _check(rc, "dsm_create")
+    return h
+
+
+def dsm_set_gamma(h, gamma: float) -> None:
+    _check(load_library().dsm_set_gamma(h, gamma), "dsm_set_gamma")
+
+
+def dsm_fill_synthetic_grads(h, step: int, stream=None) -> None:
+    _check(load_library().dsm_fill_synthetic_grads(h, step, _stream(stream)), "dsm_fill_synthetic_grads")
+
+
+def dsm_grad_ptr(h, worker: int) -> int:
+    p = c_void_p()
+    _check(load_library().dsm_grad_ptr(h, worker, byref(p)), "dsm_grad_ptr")
+    return p.value
+
+
+def dsm_load_grads(h, src_ptr: int, src_is_device: bool, stream=None) -> None:
+    _check(load_library().dsm_load_grads(h, c_void_p(src_ptr), int(bool(src_is_device)), _stream(stream)),
+           "dsm_load_grads")
+
+
+def dsm_local_step(h, stream=None) -> None:
+    _check(load_library().dsm_local_step(h, _stream(stream)), "dsm_local_step")
+
+
+def dsm_global_step(h, stream=None, stats=None) -> None:
+    """``stats``: None, or a ctypes array of dsm_tensor_stats (host) to fill (synchronises)."""
+    if stats is None:
+        rc = load_library().dsm_global_step(h, _stream(stream), None, 0)
+    else:
+        rc = load_library().dsm_global_step(h, _stream(stream), ctypes.cast(stats, POINTER(dsm_tensor_stats)),
+                                            len(stats))
+    _check(rc, "dsm_global_step")
+
+
+def dsm_stats_ptr(h) -> int:
+    p = c_void_p()
+    _check(load_library().dsm_stats_ptr(h, byref(p)), "dsm_stats_ptr")
+    return p.value
+
+
+def dsm_read_params(h, which: int, worker: int, dst_ptr: int, offset: int, count: int, dst_is_device: bool,
+                    stream=None) -> None:
+    _check(load_library().dsm_read_params(h, which, worker, c_void_p(dst_ptr), offset, count,
+                                          int(bool(dst_is_device)), _stream(stream)), "dsm_read_params")
+
+
+def dsm_write_params(h, which: int, worker: int, src_ptr: int, offset: int, count: int, src_is_device: bool,
+                     stream=None) -> None:
+    _check(load_library().dsm_write_params(h, which, worker, c_void_p(src_ptr), offset, count,
+                                           int(bool(src_is_device)), _stream(stream)), "dsm_write_params")
+
+
+def dsm_set_round(h, round_: int) -> None:
+    _check(load_library().dsm_set_round(h, round_), "dsm_set_round")
+
+
+def dsm_get_info(h) -> dsm_info:
+    info = dsm_info()
+    _check(load_library().dsm_get_info(h, byref(info)), "dsm_get_info")
+    return info
+
+
+def dsm_destroy(h) -> None:
+    _check(load_library().dsm_destroy(h), "dsm_destroy")
+
+
+# ---- convenience wrapper --------------------------------------------------
+
+class DistributedSignMomentum:
+    """One problem instance: the arena (a torch uint8 tensor on ``device``) and its handle.
+
+    tensors: objects with numel, grad_scale, kind, wd; hp: an object with
+    the dsm_hparams field names.  x0: optional float32 torch tensor of d
+    elements (host or device).
+    """
+
+    def __init__(self, tensors, n: int, tau: int, hp, device="cuda", x0=None, stream=None):
+        import torch
+        self.layout = make_layout(tensors)
+        self.hp = make_hparams(hp)
+        self.n, self.tau = int(n), int(tau)
+        self.nbytes = dsm_state_bytes(self.layout, self.n, self.hp)
+        self.device = torch.device(device)
+        raw = torch.empty(self.nbytes + 256, dtype=torch.uint8, device=self.device)
+        shift = (-raw.data_ptr()) % 256
+        self.arena = raw[shift:shift + self.nbytes]
+        self._raw = raw
+        x0_ptr, x0_dev = None, False
+        if x0 is not None:
+            x0 = x0.contiguous().to(torch.float32)
+            self._x0 = x0
+            x0_ptr, x0_dev = x0.data_ptr(), x0.is_cuda
+        with torch.cuda.device(self.device):
+            self.h = dsm_create(self.layout, self.n, self.tau, self.hp, self.arena.data_ptr(), self.nbytes,
+                                x0_ptr, x0_dev, stream)
+        info = dsm_get_info(self.h)
+        self.d, self.d_stride = int(info.d), int(info.d_stride)
+        self.num_tensors = int(info.num_tensors)
+
+    # Algorithm 1, one call per step
+    def set_gamma(self, gamma):
+        dsm_set_gamma(self.h, gamma)
+
+    def fill_synthetic_grads(self, step, stream=None):
+        dsm_fill_synthetic_grads(self.h, step, stream)
+
+    def load_grads(self, src, stream=None):
+        dsm_load_grads(self.h, src.data_ptr(), src.is_cuda, stream)
+
+    def local_step(self, stream=None):
+        dsm_local_step(self.h, stream)
+
+    def global_step(self, stream=None, with_stats=False):
+        if not with_stats:
+            dsm_global_step(self.h, stream)
+            return None
+        arr = (dsm_tensor_stats * self.num_tensors)()
+        dsm_global_step(self.h, stream, arr)
+        return [a.as_dict() for a in arr]
+
+    def synthetic_round(self, stream=None, with_stats=False):
+        """tau x (synthetic gradients + local step), then the global step."""
+        info = dsm_get_info(self.h)
+        base = int(info.round) * self.tau
+        for k in range(self.tau):
+            self.fill_synthetic_grads(base + k, stream)
+            self.local_step(stream)
+        return self.global_step(stream, with_stats)
+
+    def read(self, which, worker=0, offset=0, count=None, out=None, stream=None):
+        """Buffer `which` as a tensor (a new CPU tensor unless ``out`` is given)."""
+        import torch
+        count = self.d - offset if count is None else count
+        dt = torch.float32
+        if which == BUF_GRAD and self.hp.grad_dtype == BF16:
+            dt = torch.bfloat16
+        if out is None:
+            out = torch.empty(count, dtype=dt)
+        dsm_read_params(self.h, which, worker, out.data_ptr(), offset, count, out.is_cuda, stream)
+        return out
+
+    def write(self, which, src, worker=0, offset=0, stream=None):
+        src = src.contiguous()
+        dsm_write_params(self.h, which, worker, src.data_ptr(), offset, src.numel(), src.is_cuda, stream)
+
+    def info(self):
+        return dsm_get_info(self.h)
+
+    def close(self):
+        if getattr(self, "h", None) is not None:
+            dsm_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,69 @@
+"""Helpers shared by the GPU parity tests."""
+from __future__ import annotations
+
+import numpy as np
+
+from paper_2411_17866_gb300 import dsm
+
+# Statistics: sums are fp32 over the 8 elements of one thread (at most
+# 8 squares, or 8*n squared differences for the drift), then fp64; the
+# relative error of a sum of non-negative fp32 terms accumulated over k terms
+# is below (k+1) * 2^-24 (about 4e-6 for k = 64).  Counts are exact.
+STATS_RTOL = 1e-5
+
+
+def bits(a) -> np.ndarray:
+    a = np.ascontiguousarray(a)
+    return a.view(np.uint16 if a.dtype.itemsize == 2 else np.uint32)
+
+
+def assert_bitexact(got, want, what):
+    got = np.asarray(got)
+    want = np.asarray(want, dtype=got.dtype)
+    if not np.array_equal(bits(got), bits(want)):
+        bad = np.flatnonzero(bits(got) != bits(want))
+        i = bad[0]
+        raise AssertionError(f"{what}: {bad.size} of {got.size} elements differ; first at {i}: "
+                             f"gpu {got[i]!r} oracle {want[i]!r}")
+
+
+def compare_state(run, ora, elems=None, grads=True):
+    """Every buffer of the GPU state against the oracle, bit for bit (optionally on a subset)."""
+    import torch
+    sel = slice(None) if elems is None else elems
+
+    def rd(which, w=0):
+        t = run.read(which, w)
+        if t.dtype == torch.bfloat16:
+            t = t.to(torch.float32)
+        return t.numpy()[sel]
+
+    assert_bitexact(rd(dsm.BUF_X), ora.x, "x")
+    assert_bitexact(rd(dsm.BUF_M), ora.m, "m")
+    for i in range(ora.n):
+        assert_bitexact(rd(dsm.BUF_REPLICA, i), ora.X[i], f"replica {i}")
+        assert_bitexact(rd(dsm.BUF_OPT_M, i), ora.opt_m[i], f"opt_m {i}")
+        if ora.opt_v is not None:
+            assert_bitexact(rd(dsm.BUF_OPT_V, i), ora.opt_v[i], f"opt_v {i}")
+
+
+def compare_stats(got, want):
+    assert len(got) == len(want)
+    for T, (g, w) in enumerate(zip(got, want)):
+        for key in ("zero_sign", "flips", "unanimous", "clamped"):
+            assert g[key] == w[key], (T, key, g[key], w[key])
+        for key in ("delta_sq", "drift"):
+            assert abs(g[key] - w[key]) <= STATS_RTOL * abs(w[key]) + 1e-300, (T, key, g[key], w[key])
+
+
+def sample_elements(tensors, count, seed=0, edge=64):
+    """Sampled logical indices: the first and last `edge` elements of every tensor plus `count` random ones."""
+    rng = np.random.default_rng(seed)
+    starts = np.cumsum([0] + [t.numel for t in tensors])
+    d = int(starts[-1])
+    parts = [rng.integers(0, d, count)]
+    for a, b in zip(starts[:-1], starts[1:]):
+        if b > a:
+            parts.append(np.arange(a, min(b, a + edge)))
+            parts.append(np.arange(max(a, b - edge), b))
+    return np.unique(np.concatenate(parts)).astype(np.int64)

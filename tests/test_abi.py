@@ -1,0 +1,127 @@
+"""The C-ABI library loads, exports every declared symbol, and checks its
+arguments on the host (no GPU needed: every case fails before any CUDA call)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import workloads as W
+from paper_2411_17866_gb300 import dsm
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "dsm.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dsm_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(dsm.LIB_PATH):
+        from paper_2411_17866_gb300 import build
+        build.build()
+    return dsm.load_library()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) >= 15
+    for name in names:
+        assert hasattr(lib, name), name
+    assert set(names) == set(dsm._PROTOS), "binding and header disagree"
+
+
+def test_struct_sizes_match_header_layout():
+    assert ctypes.sizeof(dsm.dsm_tensor) == 24
+    assert ctypes.sizeof(dsm.dsm_hparams) == 72
+    assert ctypes.sizeof(dsm.dsm_tensor_stats) == 48
+
+
+def _args(tensors=None, n=4, hp=None):
+    tensors = tensors if tensors is not None else W.gpt2_layout(2, 64, 256)
+    return dsm.make_layout(tensors), n, dsm.make_hparams(hp or W.HParams())
+
+
+def test_state_bytes_covers_the_state(lib):
+    lay, n, hp = _args()
+    d = sum(t.numel for t in W.gpt2_layout(2, 64, 256))
+    nb = dsm.dsm_state_bytes(lay, n, hp)
+    # x, m, n replicas, n AdamW first and second moments, n fp32 gradients
+    assert nb >= 4 * d * (2 + 4 * n)
+    assert nb % 256 == 0
+    # bf16 gradients take half the gradient bytes; SGD-momentum drops the second moment
+    nb_bf16 = dsm.dsm_state_bytes(lay, n, dsm.make_hparams(W.HParams(grad_dtype=W.BF16)))
+    nb_sgd = dsm.dsm_state_bytes(lay, n, dsm.make_hparams(W.SGDM_HP))
+    assert nb - nb_bf16 >= 2 * d * n - 256 * 12
+    assert nb - nb_sgd >= 4 * d * n - 256 * 12
+    # grows with n
+    assert dsm.dsm_state_bytes(lay, n + 1, hp) > nb
+
+
+@pytest.mark.parametrize("bad,code", [
+    (dict(n=0), dsm.DSM_EINVAL),
+    (dict(n=65), dsm.DSM_ERANGE),
+    (dict(hp=W.HParams(lr=0.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(lr=float("nan"))), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(b1=1.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(b2=-0.1)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(eps=0.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(g_b1=1.5)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(g_eta=-1.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(sign_mode=3)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(sign_mode=W.RSIGN_ZERO, rsign_B=0.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(grad_dtype=2)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(base=7)), dsm.DSM_EINVAL),
+    (dict(hp=W.SGDM_HP.__class__(**{**W.SGDM_HP.__dict__, "mu": 1.0})), dsm.DSM_EINVAL),
+    (dict(tensors=()), dsm.DSM_EINVAL),
+    (dict(tensors=(W.Tensor("z", 0, 0, 1.0),)), dsm.DSM_EINVAL),
+    (dict(tensors=(W.Tensor("k", 8, 9, 1.0),)), dsm.DSM_EINVAL),
+])
+def test_invalid_arguments_are_rejected(lib, bad, code):
+    lay, n, hp = _args(bad.get("tensors"), bad.get("n", 4), bad.get("hp"))
+    assert lib.dsm_state_bytes(ctypes.byref(lay), n, ctypes.byref(hp)) == 0
+    h = ctypes.c_void_p(1)
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), ctypes.c_void_p(1 << 20), 1 << 40, None, 0,
+                        None, ctypes.byref(h))
+    assert rc == code, dsm.last_error()
+    assert h.value is None
+    assert dsm.last_error()
+
+
+def test_arena_checks(lib):
+    lay, n, hp = _args()
+    need = dsm.dsm_state_bytes(lay, n, hp)
+    h = ctypes.c_void_p()
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), ctypes.c_void_p((1 << 20) + 16), need, None, 0,
+                        None, ctypes.byref(h))
+    assert rc == dsm.DSM_EALIGN and "aligned" in dsm.last_error()
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), ctypes.c_void_p(1 << 20), need - 1, None, 0,
+                        None, ctypes.byref(h))
+    assert rc == dsm.DSM_ENOMEM
+    rc = lib.dsm_create(ctypes.byref(lay), n, 0, ctypes.byref(hp), ctypes.c_void_p(1 << 20), need, None, 0,
+                        None, ctypes.byref(h))
+    assert rc == dsm.DSM_EINVAL and "tau" in dsm.last_error()
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), None, need, None, 0, None, ctypes.byref(h))
+    assert rc == dsm.DSM_EINVAL
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), ctypes.c_void_p(1 << 20), need, None, 0,
+                        None, None)
+    assert rc == dsm.DSM_EINVAL
+
+
+def test_null_handle_calls_fail_cleanly(lib):
+    assert lib.dsm_local_step(None, None) == dsm.DSM_EINVAL
+    assert lib.dsm_global_step(None, None, None, 0) == dsm.DSM_EINVAL
+    assert lib.dsm_set_gamma(None, ctypes.c_float(1.0)) == dsm.DSM_EINVAL
+    assert lib.dsm_fill_synthetic_grads(None, 0, None) == dsm.DSM_EINVAL
+    assert lib.dsm_read_params(None, 0, 0, None, 0, 0, 0, None) == dsm.DSM_EINVAL
+    assert lib.dsm_destroy(None) == dsm.DSM_OK
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    monkeypatch.setattr(dsm, "_lib", None)
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        dsm.load_library(str(tmp_path / "missing.so"))

@@ -1,0 +1,245 @@
+"""GPU kernels (through the C ABI) against the CPU oracle, element by element.
+
+Tolerance: bit-exact.  The kernels evaluate the oracle's fp32 expression
+trees one rounding at a time (no contraction), with the same worker order,
+so x, m, every replica, every base-optimizer state and every gradient must
+be identical bit for bit.  The statistics' sums are compared to a relative
+1e-5 (see gpu_common.STATS_RTOL); their counts exactly.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+import workloads as W
+from gpu_common import assert_bitexact, compare_state, compare_stats, sample_elements
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from oracle import dsm_oracle as O  # noqa: E402
+from paper_2411_17866_gb300 import dsm  # noqa: E402
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    dsm.load_library()
+    yield
+    torch.cuda.empty_cache()
+
+
+# tensors whose sizes leave ragged tails and unaligned starts, and an empty tensor
+RAGGED = (W.Tensor("a", 7, W.KIND_WEIGHT, 1e-2), W.Tensor("b", 2049, W.KIND_WEIGHT, 1e-3),
+          W.Tensor("c", 8, W.KIND_BIAS, 1e-3, wd=0), W.Tensor("d", 5000, W.KIND_LN_W, 1e-3),
+          W.Tensor("e", 1, W.KIND_LN_B, 1e-3), W.Tensor("f", 0, W.KIND_WEIGHT, 1e-3),
+          W.Tensor("g", 4096, W.KIND_WEIGHT, 1e-2), W.Tensor("h", 77, W.KIND_BIAS, 1e-4),
+          W.Tensor("i", 65537, W.KIND_WEIGHT, 1e-3))
+# a small GPT-2-shaped layout: every tensor a multiple of 64 elements (vector paths)
+MINI = W.gpt2_layout(2, 64, 256)
+
+ADAMW = W.HParams()
+SGDM = W.SGDM_HP
+
+CASES = [
+    ("adamw-f32-n4-t3", ADAMW, 4, 3),
+    ("adamw-bf16-n8-t2", dataclasses.replace(ADAMW, grad_dtype=W.BF16, seed=3), 8, 2),
+    ("adamw-f32-n1-t1", ADAMW, 1, 1),
+    ("adamw-f32-n3-t2", dataclasses.replace(ADAMW, seed=7), 3, 2),
+    ("sgdm-rsign0-f32-n8-t2", SGDM, 8, 2),
+    ("sgdm-rsignpm-bf16-n2-t3", dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, grad_dtype=W.BF16), 2, 3),
+    ("sgd-plain-sign-n5-t1", dataclasses.replace(SGDM, mu=0.0, sign_mode=W.SIGN), 5, 1),
+    ("adamw-rsignpm-n9-generic", dataclasses.replace(ADAMW, sign_mode=W.RSIGN_PM, rsign_B=1.0), 9, 2),
+    ("sgdm-rsign0-n16-generic", dataclasses.replace(SGDM, seed=11), 16, 1),
+    ("adamw-n6-t2", ADAMW, 6, 2),
+    ("adamw-n7-t1", ADAMW, 7, 1),
+]
+
+
+@pytest.mark.parametrize("layout_name", ["ragged", "mini"])
+@pytest.mark.parametrize("name,hp,n,tau", CASES, ids=[c[0] for c in CASES])
+def test_rounds_bitexact(layout_name, name, hp, n, tau):
+    tensors = RAGGED if layout_name == "ragged" else MINI
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    compare_state(run, ora)
+    for t in range(2):
+        base = t * tau
+        for k in range(tau):
+            run.fill_synthetic_grads(base + k)
+            g = run.read(dsm.BUF_GRAD, n - 1)
+            ora_g = O.synthetic_grad(ora.elems, ora.scale, hp.seed, base + k, n - 1, hp.grad_dtype)
+            assert_bitexact(g.to(torch.float32).numpy(), ora_g, f"grad step {base + k}")
+            run.local_step()
+            ora.local_step()
+        stats = run.global_step(with_stats=True)
+        ora.global_step()
+        compare_state(run, ora)
+        compare_stats(stats, ora.last_stats)
+    run.close()
+
+
+def test_caller_gradients_host_and_device():
+    """dsm_load_grads: gradients written by the caller (pinned host and device)."""
+    tensors, n, tau = MINI, 3, 2
+    hp = ADAMW
+    d = sum(t.numel for t in tensors)
+    rng = np.random.default_rng(0)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp)
+    for k in range(tau):
+        g = (rng.standard_normal((n, d)) * 1e-3).astype(np.float32)
+        src = torch.from_numpy(g).pin_memory() if k == 0 else torch.from_numpy(g).cuda()
+        run.load_grads(src)
+        run.local_step()
+        ora.local_step([g[i] for i in range(n)])
+    run.global_step()
+    ora.global_step()
+    compare_state(run, ora)
+    run.close()
+
+
+def test_order_of_algorithm_1_is_enforced():
+    run = dsm.DistributedSignMomentum(MINI, 2, 2, ADAMW)
+    with pytest.raises(dsm.DsmError) as e:
+        run.global_step()
+    assert e.value.code == dsm.DSM_ESTATE
+    run.fill_synthetic_grads(0)
+    run.local_step()
+    with pytest.raises(dsm.DsmError) as e:
+        run.set_gamma(1e-3)
+    assert e.value.code == dsm.DSM_ESTATE
+    run.local_step()
+    with pytest.raises(dsm.DsmError) as e:
+        run.local_step()
+    assert e.value.code == dsm.DSM_ESTATE
+    run.global_step()
+    with pytest.raises(dsm.DsmError) as e:
+        run.read(dsm.BUF_REPLICA, worker=2)
+    assert e.value.code == dsm.DSM_ERANGE
+    with pytest.raises(dsm.DsmError) as e:
+        run.read(dsm.BUF_X, offset=run.d, count=1)
+    assert e.value.code == dsm.DSM_ERANGE
+    run.close()
+
+
+def test_gamma_schedule():
+    """A different gamma_t each round (e.g. a cosine schedule) reaches the local and global steps."""
+    tensors, n, tau = MINI, 2, 2
+    run = dsm.DistributedSignMomentum(tensors, n, tau, ADAMW)
+    ora = O.OracleRun(tensors, n, tau, ADAMW)
+    for gamma in (6e-4, 3e-4, 1.5e-4):
+        run.set_gamma(gamma)
+        ora.gamma = gamma
+        run.synthetic_round()
+        ora.run_round()
+    compare_state(run, ora)
+    run.close()
+
+
+def test_checkpoint_resume_bitexact():
+    tensors, n, tau = MINI, 4, 2
+    hp = dataclasses.replace(SGDM, sign_mode=W.RSIGN_ZERO)
+    a = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    a.synthetic_round()
+    bufs = [(dsm.BUF_X, 0), (dsm.BUF_M, 0)] + [(b, i) for i in range(n) for b in (dsm.BUF_REPLICA, dsm.BUF_OPT_M)]
+    saved = [(b, i, a.read(b, i).clone()) for b, i in bufs]
+    b = dsm.DistributedSignMomentum(tensors, n, tau, hp, x0=torch.zeros(a.d))
+    for which, i, v in saved:
+        b.write(which, v, worker=i)
+    dsm.dsm_set_round(b.h, 1)
+    a.synthetic_round()
+    b.synthetic_round()
+    torch.cuda.synchronize()
+    for which, i in bufs:
+        assert torch.equal(a.read(which, i), b.read(which, i))
+    a.close()
+    b.close()
+
+
+def test_deterministic_statistics():
+    tensors, n, tau = MINI, 4, 2
+    outs = []
+    for _ in range(2):
+        run = dsm.DistributedSignMomentum(tensors, n, tau, ADAMW)
+        outs.append(run.synthetic_round(with_stats=True))
+        run.close()
+    assert outs[0] == outs[1]
+
+
+def test_x0_from_device_and_host():
+    tensors, n, tau = MINI, 2, 1
+    d = sum(t.numel for t in tensors)
+    x0 = torch.linspace(-1, 1, d, dtype=torch.float32)
+    for src in (x0, x0.cuda()):
+        run = dsm.DistributedSignMomentum(tensors, n, tau, ADAMW, x0=src)
+        ora = O.OracleRun(tensors, n, tau, ADAMW, x0=x0.numpy())
+        compare_state(run, ora)
+        run.synthetic_round()
+        ora.run_round()
+        compare_state(run, ora)
+        run.close()
+
+
+@pytest.mark.parametrize("key", list(W.WORKLOADS))
+def test_full_workloads_sampled(key):
+    """Each measured workload at full size, one round, in the launch sequence the benchmark uses,
+    checked on sampled elements against the element-subset oracle (first and last 64 elements of
+    every tensor plus 20000 random ones; the whole model for the flat workload)."""
+    wl = W.WORKLOADS[key]
+    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, wl.hp)
+    elems = None if wl.d <= (1 << 20) else sample_elements(wl.tensors, 20000)
+    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=elems, with_stats=elems is None)
+    rounds = wl.rounds if elems is None else 1
+    for _ in range(rounds):
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+    torch.cuda.synchronize()
+    sel = None if elems is None else torch.from_numpy(elems).cuda()
+    buf = torch.empty(wl.d, dtype=torch.float32, device="cuda")
+
+    def rd(which, i=0):
+        run.read(which, i, out=buf)
+        return (buf if sel is None else buf[sel]).cpu().numpy()
+
+    assert_bitexact(rd(dsm.BUF_X), ora.x, "x")
+    assert_bitexact(rd(dsm.BUF_M), ora.m, "m")
+    for i in range(wl.n):
+        assert_bitexact(rd(dsm.BUF_REPLICA, i), ora.X[i], f"replica {i}")
+        assert_bitexact(rd(dsm.BUF_OPT_M, i), ora.opt_m[i], f"opt_m {i}")
+        if ora.opt_v is not None:
+            assert_bitexact(rd(dsm.BUF_OPT_V, i), ora.opt_v[i], f"opt_v {i}")
+    if elems is None:
+        compare_stats(stats, ora.last_stats)
+    else:
+        # properties that hold at any size
+        assert sum(s["unanimous"] for s in stats) <= wl.d
+        assert all(s["delta_sq"] > 0 for s in stats)
+    run.close()
+    del run
+    torch.cuda.empty_cache()
+
+
+def test_fp64_twin_within_stated_tolerance():
+    """The GPU result against the fp64 oracle: |x - x64| <= 1e-6 (1 + |x|); sign mismatches only
+    where |u| <= 1e-6 max|u|, counted."""
+    wl = W.WORKLOADS["flat1m"]
+    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, wl.hp)
+    elems = np.arange(0, wl.d, 7)
+    ora64 = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=elems, dtype=np.float64)
+    diverged = np.zeros(elems.size, dtype=bool)
+    mismatches = 0
+    for _ in range(wl.rounds):
+        run.synthetic_round()
+        ora64.run_round()
+        u64 = ora64.last_inter["u"]
+        x = run.read(dsm.BUF_X).numpy()[elems].astype(np.float64)
+        # an element whose sign differs from the fp64 twin moves by 2*eta*gamma; find them
+        moved = np.abs(x - ora64.x) > 1e-6 * (1 + np.abs(ora64.x))
+        near_zero = np.abs(u64) <= 1e-6 * np.max(np.abs(u64))
+        assert np.all(near_zero[moved & ~diverged])
+        mismatches += int(np.sum(moved & ~diverged))
+        diverged |= moved
+    print(f"sign mismatches vs fp64: {mismatches} of {elems.size}")
+    run.close()
