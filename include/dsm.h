@@ -237,6 +237,54 @@ int dsm_destroy(dsm_handle* h);
 /* Message for the calling thread's last failed call ("" if none). */
 const char* dsm_last_error(void);
 
+/* ---- global step without any device allocation ----------------------- */
+/* The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory themselves: code that lives inside a
+ * host framework which owns all of HBM through its own pool allocator and
+ * forbids outside allocations, or latency-critical loops in which a
+ * cudaMalloc/cudaFree (which may block or synchronise the device) is not
+ * acceptable.  Such a caller has its model, momentum and replicas in
+ * buffers it already owns, but no arena for dsm_create().
+ *
+ * dsm_global_step_noalloc() runs the same global step as dsm_global_step()
+ * (same kernels, bit-identical results) directly on the caller's buffers.
+ * Its tile table and per-tile statistics live in one scratch array inside
+ * the library, a static device array of DSM_NOALLOC_SCRATCH_BYTES bytes that
+ * every GPU which loads the library holds until the process exits.  Nothing
+ * is allocated: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * Limits: at most DSM_NOALLOC_MAX_TENSORS tensors and DSM_NOALLOC_MAX_TILES
+ * tiles of 2048 elements (a one-tensor model of up to 2^30 elements); larger
+ * layouts return DSM_ERANGE.
+ *
+ * Arguments: layout, n (1..64) and hp as for dsm_create (only the global
+ * fields of hp and its seed are used); gamma the round's gamma_t (> 0);
+ * round the round index t (it keys the randomized sign); x and m the global
+ * model and momentum (d fp32 each, device); replicas the n worker models
+ * (device, fp32, worker i at replicas + i*replica_stride, replica_stride >= d
+ * and a multiple of 8); x, m and replicas 16-byte aligned.  x, m and the
+ * replicas are updated in place.  stats: NULL, or num_tensors entries in
+ * device memory (stats_is_device = 1) or host memory (0; the call then
+ * synchronises the stream).  Runs on the current device, which must own
+ * the buffers.
+ *
+ * The first call on a device looks up the scratch array's device address
+ * (cudaGetSymbolAddress) and caches it; make that first call before any
+ * stream capture.  All calls share the one scratch array and leave their
+ * contents in it; nothing in it needs to start at zero, because every call
+ * rewrites the parts it reads.  Calls whose work overlaps on the GPU (on
+ * different streams, or from different threads, on the same device) race
+ * on the scratch array: order them on one stream or serialise them.  The
+ * layout's tensor list is copied to the device on the stream; from pageable
+ * host memory that copy has consumed the list when the call returns, from
+ * pinned memory the list must stay unchanged until the stream reaches it. */
+#define DSM_NOALLOC_MAX_TENSORS 4096u
+#define DSM_NOALLOC_MAX_TILES   524288u
+#define DSM_NOALLOC_SCRATCH_BYTES 25657344u
+int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp, float gamma,
+                            uint64_t round, float* x, float* m, float* replicas, uint64_t replica_stride,
+                            dsm_tensor_stats* stats, int stats_is_device, dsm_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -152,6 +152,8 @@ struct DeviceGuard {
 
 }  // namespace
 
+void dsm::set_last_error_message(const char* msg) { g_last_error = msg; }
+
 struct dsm_handle {
     int device = 0;
     uint32_t n = 0, tau = 0;

@@ -120,4 +120,7 @@ cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const Sgd
 cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);
 cudaError_t launch_stats(const Problem& p, cudaStream_t s);
 
+// Sets the calling thread's message returned by dsm_last_error() (dsm_api.cpp).
+void set_last_error_message(const char* msg);
+
 }  // namespace dsm

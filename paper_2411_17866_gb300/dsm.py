@@ -81,6 +81,9 @@ _PROTOS = {
     "dsm_get_info": (c_int, [c_void_p, POINTER(dsm_info)]),
     "dsm_destroy": (c_int, [c_void_p]),
     "dsm_last_error": (c_char_p, []),
+    "dsm_global_step_noalloc": (c_int, [POINTER(dsm_layout), c_uint32, POINTER(dsm_hparams), c_float, c_uint64,
+                                        c_void_p, c_void_p, c_void_p, c_uint64, POINTER(dsm_tensor_stats), c_int,
+                                        c_void_p]),
 }
 
 _lib = None
@@ -229,6 +232,23 @@ def dsm_get_info(h) -> dsm_info:
 
 def dsm_destroy(h) -> None:
     _check(load_library().dsm_destroy(h), "dsm_destroy")
+
+
+def dsm_global_step_noalloc(layout, n, hp, gamma, round_, x_ptr, m_ptr, replicas_ptr, replica_stride,
+                            stats=None, stats_is_device=False, stream=None) -> None:
+    """The global step on caller-owned device buffers, with the library's static scratch array
+    (for callers that cannot allocate device memory).  ``stats``: None, a ctypes array of
+    dsm_tensor_stats in host memory, or a device address (int) with stats_is_device=True."""
+    if stats is None:
+        sp = None
+    elif stats_is_device:
+        sp = ctypes.cast(c_void_p(stats), POINTER(dsm_tensor_stats))
+    else:
+        sp = ctypes.cast(stats, POINTER(dsm_tensor_stats))
+    rc = load_library().dsm_global_step_noalloc(byref(layout), n, byref(hp), gamma, round_, c_void_p(x_ptr),
+                                                c_void_p(m_ptr), c_void_p(replicas_ptr), replica_stride, sp,
+                                                int(bool(stats_is_device)), _stream(stream))
+    _check(rc, "dsm_global_step_noalloc")
 
 
 # ---- convenience wrapper --------------------------------------------------
