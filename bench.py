@@ -51,7 +51,38 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    # smaller cases of a workload (profiling captures): fewer workers, fewer local steps, or a
+    # prefix of the tensor list holding at most this many parameters
+    ap.add_argument("--n-workers", type=int, default=None)
+    ap.add_argument("--tau", type=int, default=None)
+    ap.add_argument("--max-params", type=int, default=None)
     return ap.parse_args()
+
+
+def select_workload(args):
+    import dataclasses
+    wl = W.WORKLOADS[args.workload]
+    changes = {}
+    notes = []
+    if args.n_workers:
+        changes["n"] = args.n_workers
+        notes.append(f"n={args.n_workers}")
+    if args.tau:
+        changes["tau"] = args.tau
+        notes.append(f"tau={args.tau}")
+    if args.max_params:
+        keep, total = [], 0
+        for t in wl.tensors:
+            if keep and total + t.numel > args.max_params:
+                break
+            keep.append(t)
+            total += t.numel
+        changes["tensors"] = tuple(keep)
+        notes.append(f"first {len(keep)} tensors ({total} params)")
+    if changes:
+        changes["name"] = wl.name + " [reduced: " + ", ".join(notes) + "]"
+        wl = dataclasses.replace(wl, **changes)
+    return wl
 
 
 def dist_env():
@@ -171,7 +202,7 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
-    wl = W.WORKLOADS[args.workload]
+    wl = select_workload(args)
     import numpy as np
 
     from oracle import dsm_oracle as O
@@ -220,7 +251,7 @@ def main():
         dist.init_process_group("gloo", rank=rank, world_size=world)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    wl = W.WORKLOADS[args.workload]
+    wl = select_workload(args)
     import dataclasses
     hp = dataclasses.replace(wl.hp, seed=wl.hp.seed + rank)
     run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp, device=dev)
