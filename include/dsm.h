@@ -128,8 +128,10 @@ typedef struct {
  *   flips     = #{e : sign(u_e) != sign(Delta_e)}                    (momentum overrides the round's direction)
  *   unanimous = #{e : sign(x_e - x_{i,e}) = sign(Delta_e) for every worker i}
  *   clamped   = #{e : |u_e| > B} in the randomized modes, else 0
- * Sums are accumulated in fp32 over the 8 elements of one thread and in
- * fp64 beyond (relative error below 1e-5); counts are exact. */
+ * Per element the terms are fp32 values; they are summed with compensated
+ * (TwoSum) fp32 arithmetic per thread and warp and in fp64 beyond, so a
+ * tensor's sums are within (n + 2) * 2^-24 relative of the exact sums of
+ * the element terms; counts are exact. */
 typedef struct {
     double delta_sq;
     double drift;
@@ -254,7 +256,7 @@ const char* dsm_last_error(void);
  * is allocated: no cudaMalloc, no cudaFree, no allocating library routine.
  *
  * Limits: at most DSM_NOALLOC_MAX_TENSORS tensors and DSM_NOALLOC_MAX_TILES
- * tiles of 2048 elements (a one-tensor model of up to 2^30 elements); larger
+ * tiles of 1024 elements (a one-tensor model of up to 2^29 elements); larger
  * layouts return DSM_ERANGE.
  *
  * Arguments: layout, n (1..64) and hp as for dsm_create (only the global

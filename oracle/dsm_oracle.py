@@ -85,10 +85,16 @@ def hash_key(seed: int, stream: int, idx: int):
 
 
 def hash24(seed: int, stream: int, idx: int, elems):
-    """24-bit draw of element e: top 24 bits of output e+1 of SplitMix64(key(seed, stream, idx))."""
+    """24-bit draw of element e from SplitMix64(key(seed, stream, idx)).
+
+    Each 64-bit output serves two consecutive elements: output floor(e/2)+1
+    gives bits 63..40 to the even element and bits 39..16 to the odd one.
+    """
     key = hash_key(seed, stream, idx)
     e = np.asarray(elems, dtype=U64)
-    return splitmix64_output(np.full(e.shape, key, dtype=U64), e + U64(1)) >> U64(40)
+    h = splitmix64_output(np.full(e.shape, key, dtype=U64), (e >> U64(1)) + U64(1))
+    shift = np.where((e & U64(1)) == 0, U64(40), U64(16))
+    return (h >> shift) & U64(0xFFFFFF)
 
 
 def uniform24(seed: int, stream: int, idx: int, elems) -> np.ndarray:

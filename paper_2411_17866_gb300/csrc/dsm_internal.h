@@ -11,10 +11,11 @@ namespace dsm {
 
 // Elements of one tile.  A tile lies inside one tensor; a tensor of numel
 // elements has ceil(numel / kTile) tiles.  One CTA of kThreads threads
-// processes one tile, kElemsPerThread consecutive elements per thread.
+// processes one tile, kElemsPerThread consecutive elements per thread (one
+// 16-byte vector of every fp32 stream).
 constexpr uint32_t kThreads = 256;
-constexpr uint32_t kElemsPerThread = 8;
-constexpr uint32_t kTile = kThreads * kElemsPerThread;  // 2048
+constexpr uint32_t kElemsPerThread = 4;
+constexpr uint32_t kTile = kThreads * kElemsPerThread;  // 1024
 constexpr uint32_t kMaxWorkers = 64;
 constexpr uint32_t kMaxUnrolledWorkers = 8;  // replicas held in registers by the global step
 

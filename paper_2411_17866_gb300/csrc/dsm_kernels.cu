@@ -1,12 +1,17 @@
 // CUDA kernels (sm_103a) for one global round of distributed sign momentum
 // with local steps (arXiv 2411.17866, Algorithm 1).
 //
-// Every kernel is a persistent, grid-stride loop over tiles of at most
-// kTile = 2048 elements that lie inside one tensor.  A CTA of 256 threads
-// takes one tile at a time; each thread owns 8 consecutive elements and
-// moves them with 16-byte loads and stores (two per fp32 stream, one per
-// bf16 stream).  The work is streaming and elementwise, so it is bound by
-// HBM bandwidth; nothing here is a contraction, and no tensor core is used.
+// Every kernel is a persistent, grid-stride loop over work items: tiles of
+// at most kTile = 1024 elements that lie inside one tensor (for the local
+// steps, a tile of one worker).  A CTA of 256 threads takes one item at a
+// time; each thread owns 4 consecutive elements and moves them with one
+// 16-byte load or store per fp32 stream (8 bytes per bf16 stream), so every
+// warp instruction covers 512 contiguous bytes.  The local and global steps
+// double-buffer in registers: a thread issues the loads of its next item
+// before it computes the current one, so the HBM requests of one item are in
+// flight during the arithmetic of the previous one.  The work is streaming and
+// elementwise, bound by HBM bandwidth; nothing is a contraction, and no tensor
+// core is used.
 //
 // All method arithmetic uses the explicit round-to-nearest intrinsics
 // (__fadd_rn, __fmul_rn, __fdiv_rn, __fsqrt_rn, ...), which the compiler
@@ -28,6 +33,7 @@ namespace {
 // seeded with `state` is the state advanced j times by the golden-ratio
 // increment, passed through Stafford's variant-13 finaliser.
 constexpr uint64_t kGoldenGamma = 0x9E3779B97F4A7C15ull;
+constexpr float kTwoPowM24 = 5.9604644775390625e-08f;  // 2^-24
 
 __device__ __forceinline__ uint64_t sm64_finalise(uint64_t z) {
     z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
@@ -35,10 +41,23 @@ __device__ __forceinline__ uint64_t sm64_finalise(uint64_t z) {
     return z ^ (z >> 31);
 }
 
-// u = top 24 bits of output e+1 of SplitMix64(key), times 2^-24 (exact in fp32).
+__device__ __forceinline__ uint64_t sm64_output(uint64_t key, uint64_t j) {
+    return sm64_finalise(key + j * kGoldenGamma);
+}
+
+// The two 24-bit draws of one output: bits 63..40 (even element) and
+// 39..16 (odd element), each times 2^-24 (exact in fp32).
+__device__ __forceinline__ float draw_even(uint64_t h) {
+    return __fmul_rn(__uint2float_rn(static_cast<uint32_t>(h >> 40)), kTwoPowM24);
+}
+__device__ __forceinline__ float draw_odd(uint64_t h) {
+    return __fmul_rn(__uint2float_rn(static_cast<uint32_t>(h >> 16) & 0xFFFFFFu), kTwoPowM24);
+}
+
+// u of element e: output floor(e/2)+1 of SplitMix64(key), field by parity.
 __device__ __forceinline__ float hash_uniform(uint64_t key, uint64_t e) {
-    const uint64_t h = sm64_finalise(key + (e + 1ull) * kGoldenGamma) >> 40;
-    return __fmul_rn(__uint2float_rn(static_cast<uint32_t>(h)), 5.9604644775390625e-08f);
+    const uint64_t h = sm64_output(key, (e >> 1) + 1);
+    return (e & 1) ? draw_odd(h) : draw_even(h);
 }
 
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC 2011): ten rounds of the
@@ -67,44 +86,42 @@ __device__ __forceinline__ uint32_t word_of(const uint4& b, uint32_t i) {
 
 // r = (word >> 8) * 2^-24, exact in fp32.
 __device__ __forceinline__ float philox_unit(uint32_t w) {
-    return __fmul_rn(__uint2float_rn(w >> 8), 5.9604644775390625e-08f);
+    return __fmul_rn(__uint2float_rn(w >> 8), kTwoPowM24);
 }
 
 // ---------------------------------------------------------------------------
-// 16-byte streaming memory access
+// 16-byte streaming memory access (4 elements per thread)
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+__device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
     const float4 a = __ldcs(reinterpret_cast<const float4*>(p));
-    const float4 b = __ldcs(reinterpret_cast<const float4*>(p) + 1);
     v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 
-__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+__device__ __forceinline__ void store4(float* p, const float (&v)[4]) {
     __stcs(reinterpret_cast<float4*>(p), make_float4(v[0], v[1], v[2], v[3]));
-    __stcs(reinterpret_cast<float4*>(p) + 1, make_float4(v[4], v[5], v[6], v[7]));
 }
 
-__device__ __forceinline__ void load8_bf16(const __nv_bfloat16* p, float (&v)[8]) {
-    const uint4 raw = __ldcs(reinterpret_cast<const uint4*>(p));
-    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {  // bf16 -> fp32 is exact: the bf16 bits are the top half
-        v[2 * i] = __uint_as_float(w[i] << 16);
-        v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-    }
+// bf16 -> fp32 is exact: the bf16 bits are the top half of the fp32 encoding.
+__device__ __forceinline__ void load4_bf16(const __nv_bfloat16* p, float (&v)[4]) {
+    const uint2 raw = __ldcs(reinterpret_cast<const uint2*>(p));
+    v[0] = __uint_as_float(raw.x << 16);
+    v[1] = __uint_as_float(raw.x & 0xFFFF0000u);
+    v[2] = __uint_as_float(raw.y << 16);
+    v[3] = __uint_as_float(raw.y & 0xFFFF0000u);
 }
 
-__device__ __forceinline__ void store8_bf16(__nv_bfloat16* p, const float (&v)[8]) {
-    uint32_t w[4];
+__device__ __forceinline__ void store4_bf16(__nv_bfloat16* p, const float (&v)[4]) {
+    uint32_t h[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(v[2 * i]));
-        const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(v[2 * i + 1]));
-        w[i] = lo | (hi << 16);
-    }
-    __stcs(reinterpret_cast<uint4*>(p), make_uint4(w[0], w[1], w[2], w[3]));
+    for (int i = 0; i < 4; ++i) h[i] = __bfloat16_as_ushort(__float2bfloat16_rn(v[i]));
+    __stcs(reinterpret_cast<uint2*>(p), make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16)));
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void load4_grad(const void* g, uint64_t i, float (&v)[4]) {
+    if (kBf16) load4_bf16(reinterpret_cast<const __nv_bfloat16*>(g) + i, v);
+    else load4(reinterpret_cast<const float*>(g) + i, v);
 }
 
 __device__ __forceinline__ float load_grad1(const void* g, int bf16, uint64_t i) {
@@ -112,11 +129,12 @@ __device__ __forceinline__ float load_grad1(const void* g, int bf16, uint64_t i)
     return reinterpret_cast<const float*>(g)[i];
 }
 
-// A thread's 8 elements take the vector path when the tile start is
-// 8-element aligned (so every stream is 16-byte aligned) and all 8 lie in
-// the tile; otherwise the thread handles its elements one at a time.
+// A thread's 4 elements take the vector path when the tile start is
+// 4-element aligned (every fp32 stream 16-byte aligned, every bf16 stream
+// 8-byte aligned) and all 4 lie in the tile; otherwise the thread handles
+// its elements one at a time.
 __device__ __forceinline__ bool vector_ok(const TileDesc& td, uint32_t e0) {
-    return (td.start & 7u) == 0 && e0 + kElemsPerThread <= td.len;
+    return (td.start & 3u) == 0 && e0 + kElemsPerThread <= td.len;
 }
 
 // ---------------------------------------------------------------------------
@@ -160,8 +178,28 @@ __device__ __forceinline__ float applied_sign(float u, const GlobalScalars& g, f
     return r < q ? s : -s;
 }
 
+// Compensated fp32 sum (hi + lo): each addition keeps its rounding error
+// (Knuth's TwoSum, six fp32 operations), so long sums stay accurate to about
+// 2^-44 relative without using the fp64 pipe.
+struct CSum {
+    float hi = 0.f, lo = 0.f;
+};
+
+__device__ __forceinline__ void csum_add(CSum& s, float v) {
+    const float t = __fadd_rn(s.hi, v);
+    const float bp = __fsub_rn(t, s.hi);
+    const float err = __fadd_rn(__fsub_rn(s.hi, __fsub_rn(t, bp)), __fsub_rn(v, bp));
+    s.lo = __fadd_rn(s.lo, err);
+    s.hi = t;
+}
+
+__device__ __forceinline__ void csum_merge(CSum& a, const CSum& b) {
+    csum_add(a, b.hi);
+    a.lo = __fadd_rn(a.lo, b.lo);
+}
+
 struct ThreadStats {
-    float dsq = 0.f, drift = 0.f;
+    CSum dsq, drift;
     uint32_t zero = 0, flips = 0, unanimous = 0, clamped = 0;
 };
 
@@ -182,7 +220,7 @@ __device__ __forceinline__ void global_elem(float& x, float& m, const float (&di
     const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
     // statistics
     const int sD = sgn(D);
-    st.dsq = __fadd_rn(st.dsq, __fmul_rn(D, D));
+    csum_add(st.dsq, __fmul_rn(D, D));
     bool unan = true;
     float dr = 0.f;
 #pragma unroll
@@ -193,7 +231,7 @@ __device__ __forceinline__ void global_elem(float& x, float& m, const float (&di
             unan = unan && (sgn(dif[i]) == sD);
         }
     }
-    st.drift = __fadd_rn(st.drift, dr);
+    csum_add(st.drift, dr);
     st.zero += (s == 0.f);
     st.flips += (sgn(u) != sD);
     st.unanimous += unan;
@@ -202,16 +240,22 @@ __device__ __forceinline__ void global_elem(float& x, float& m, const float (&di
     m = mn;
 }
 
-// Fixed-order CTA reduction of the per-thread statistics into one partial.
+// Fixed-order CTA reduction of the per-thread statistics into one partial:
+// compensated fp32 across the lanes of a warp, fp64 across the warps.
 __device__ __forceinline__ void reduce_stats(const ThreadStats& st, StatPartial* out) {
     __shared__ double s_d[kThreads / 32][2];
     __shared__ uint32_t s_c[kThreads / 32][4];
-    double a = static_cast<double>(st.dsq), b = static_cast<double>(st.drift);
+    CSum a = st.dsq, b = st.drift;
     uint32_t c0 = st.zero, c1 = st.flips, c2 = st.unanimous, c3 = st.clamped;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-        a += __shfl_down_sync(0xffffffffu, a, off);
-        b += __shfl_down_sync(0xffffffffu, b, off);
+        CSum oa, ob;
+        oa.hi = __shfl_down_sync(0xffffffffu, a.hi, off);
+        oa.lo = __shfl_down_sync(0xffffffffu, a.lo, off);
+        ob.hi = __shfl_down_sync(0xffffffffu, b.hi, off);
+        ob.lo = __shfl_down_sync(0xffffffffu, b.lo, off);
+        csum_merge(a, oa);
+        csum_merge(b, ob);
         c0 += __shfl_down_sync(0xffffffffu, c0, off);
         c1 += __shfl_down_sync(0xffffffffu, c1, off);
         c2 += __shfl_down_sync(0xffffffffu, c2, off);
@@ -219,35 +263,31 @@ __device__ __forceinline__ void reduce_stats(const ThreadStats& st, StatPartial*
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
-        s_d[warp][0] = a; s_d[warp][1] = b;
+        s_d[warp][0] = static_cast<double>(a.hi) + static_cast<double>(a.lo);
+        s_d[warp][1] = static_cast<double>(b.hi) + static_cast<double>(b.lo);
         s_c[warp][0] = c0; s_c[warp][1] = c1; s_c[warp][2] = c2; s_c[warp][3] = c3;
     }
     __syncthreads();
-    if (warp == 0) {
-        constexpr int kWarps = kThreads / 32;
-        a = lane < kWarps ? s_d[lane][0] : 0.0;
-        b = lane < kWarps ? s_d[lane][1] : 0.0;
-        c0 = lane < kWarps ? s_c[lane][0] : 0u;
-        c1 = lane < kWarps ? s_c[lane][1] : 0u;
-        c2 = lane < kWarps ? s_c[lane][2] : 0u;
-        c3 = lane < kWarps ? s_c[lane][3] : 0u;
-#pragma unroll
-        for (int off = kWarps / 2; off > 0; off >>= 1) {
-            a += __shfl_down_sync(0xffffffffu, a, off);
-            b += __shfl_down_sync(0xffffffffu, b, off);
-            c0 += __shfl_down_sync(0xffffffffu, c0, off);
-            c1 += __shfl_down_sync(0xffffffffu, c1, off);
-            c2 += __shfl_down_sync(0xffffffffu, c2, off);
-            c3 += __shfl_down_sync(0xffffffffu, c3, off);
+    if (threadIdx.x == 0) {
+        StatPartial p;
+        p.delta_sq = 0.0; p.drift = 0.0;
+        p.zero_sign = p.flips = p.unanimous = p.clamped = 0;
+        for (int w = 0; w < kThreads / 32; ++w) {
+            p.delta_sq += s_d[w][0]; p.drift += s_d[w][1];
+            p.zero_sign += s_c[w][0]; p.flips += s_c[w][1]; p.unanimous += s_c[w][2]; p.clamped += s_c[w][3];
         }
-        if (lane == 0) {
-            StatPartial p;
-            p.delta_sq = a; p.drift = b;
-            p.zero_sign = c0; p.flips = c1; p.unanimous = c2; p.clamped = c3;
-            *out = p;
-        }
+        *out = p;
     }
-    __syncthreads();  // the shared arrays are reused by the next tile
+    __syncthreads();  // the shared arrays are reused by the next reduction
+}
+
+__device__ __forceinline__ void zero_partial(StatPartial* out) {
+    if (threadIdx.x == 0) {
+        StatPartial p;
+        p.delta_sq = 0.0; p.drift = 0.0;
+        p.zero_sign = p.flips = p.unanimous = p.clamped = 0;
+        *out = p;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -280,26 +320,29 @@ __global__ void __launch_bounds__(kThreads) k_init(Problem p, uint64_t key_init,
     }
 }
 
-// K1: synthetic gradients of one local step for every worker.
+// K1: synthetic gradients of one local step for every worker.  Bound by the
+// integer work of the hash (one 64-bit SplitMix64 output per two elements
+// and per draw family), not by its write stream.
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
     for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
         const TileDesc td = p.tiles[ti];
         const TensorDesc& T = p.tensors[td.tensor];
         const float s = T.scale, s2 = T.scale2;
-        const uint32_t e0 = threadIdx.x * kElemsPerThread;
         if (vector_ok(td, e0)) {
-            const uint64_t gi = td.start + e0;
-            float a[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) a[j] = step_term(s, hash_uniform(k.step, gi + j));
+            const uint64_t gi = td.start + e0;  // even: elements gi..gi+3 use outputs gi/2+1, gi/2+2
+            const uint64_t j = (gi >> 1) + 1;
+            const uint64_t h0 = sm64_output(k.step, j), h1 = sm64_output(k.step, j + 1);
+            const float a[4] = {step_term(s, draw_even(h0)), step_term(s, draw_odd(h0)),
+                                step_term(s, draw_even(h1)), step_term(s, draw_odd(h1))};
             for (uint32_t w = 0; w < p.n; ++w) {
-                float g[8];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) g[j] = grad_value(a[j], s2, hash_uniform(k.worker[w], gi + j));
+                const uint64_t q0 = sm64_output(k.worker[w], j), q1 = sm64_output(k.worker[w], j + 1);
+                const float g[4] = {grad_value(a[0], s2, draw_even(q0)), grad_value(a[1], s2, draw_odd(q0)),
+                                    grad_value(a[2], s2, draw_even(q1)), grad_value(a[3], s2, draw_odd(q1))};
                 const uint64_t o = w * p.d_stride + gi;
-                if (kBf16) store8_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
-                else store8(reinterpret_cast<float*>(p.grad) + o, g);
+                if (kBf16) store4_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
+                else store4(reinterpret_cast<float*>(p.grad) + o, g);
             }
         } else {
             const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
@@ -317,151 +360,228 @@ __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
     }
 }
 
-// K2: one AdamW local step on every worker (work item = (worker, tile)).
+// Where a local-step work item (worker w, tile) lives.
+struct LocalItem {
+    uint64_t base;   // w * d_stride + tile start
+    uint32_t len;
+    float lam;
+    bool vec;
+};
+
+__device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t item, uint32_t e0, bool local_lam) {
+    const uint32_t w = item / p.num_tiles;
+    const TileDesc td = p.tiles[item - w * p.num_tiles];
+    LocalItem it;
+    it.base = w * p.d_stride + td.start;
+    it.len = td.len;
+    it.lam = local_lam ? p.tensors[td.tensor].lam_local : 0.f;
+    it.vec = vector_ok(td, e0);
+    return it;
+}
+
+// K2: one AdamW local step on every worker (work item = (worker, tile)),
+// double-buffered in registers.
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars a) {
     const uint32_t items = p.num_tiles * p.n;
-    for (uint32_t item = blockIdx.x; item < items; item += gridDim.x) {
-        const uint32_t w = item / p.num_tiles;
-        const uint32_t ti = item - w * p.num_tiles;
-        const TileDesc td = p.tiles[ti];
-        const float lam = p.tensors[td.tensor].lam_local;
-        const uint64_t base = w * p.d_stride + td.start;
-        const uint32_t e0 = threadIdx.x * kElemsPerThread;
-        if (vector_ok(td, e0)) {
-            float x[8], m[8], v[8], g[8];
-            load8(p.X + base + e0, x);
-            load8(p.opt_m + base + e0, m);
-            load8(p.opt_v + base + e0, v);
-            if (kBf16) load8_bf16(reinterpret_cast<const __nv_bfloat16*>(p.grad) + base + e0, g);
-            else load8(reinterpret_cast<const float*>(p.grad) + base + e0, g);
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+    uint32_t item = blockIdx.x;
+    if (item >= items) return;
+    LocalItem nx = local_item(p, item, e0, true);
+    float x[4], m[4], v[4], g[4];
+    if (nx.vec) {
+        load4(p.X + nx.base + e0, x);
+        load4(p.opt_m + nx.base + e0, m);
+        load4(p.opt_v + nx.base + e0, v);
+        load4_grad<kBf16>(p.grad, nx.base + e0, g);
+    }
+    for (; item < items; item += gridDim.x) {
+        const LocalItem cur = nx;
+        float cx[4], cm[4], cv[4], cg[4];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) adamw_elem(x[j], m[j], v[j], g[j], a, lam);
-            store8(p.X + base + e0, x);
-            store8(p.opt_m + base + e0, m);
-            store8(p.opt_v + base + e0, v);
+        for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cm[j] = m[j]; cv[j] = v[j]; cg[j] = g[j]; }
+        const uint32_t next = item + gridDim.x;
+        if (next < items) {  // issue the next item's loads before computing this one
+            nx = local_item(p, next, e0, true);
+            if (nx.vec) {
+                load4(p.X + nx.base + e0, x);
+                load4(p.opt_m + nx.base + e0, m);
+                load4(p.opt_v + nx.base + e0, v);
+                load4_grad<kBf16>(p.grad, nx.base + e0, g);
+            }
+        }
+        if (cur.vec) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) adamw_elem(cx[j], cm[j], cv[j], cg[j], a, cur.lam);
+            store4(p.X + cur.base + e0, cx);
+            store4(p.opt_m + cur.base + e0, cm);
+            store4(p.opt_v + cur.base + e0, cv);
         } else {
-            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
-                const uint64_t i = base + e;
-                float x = p.X[i], m = p.opt_m[i], v = p.opt_v[i];
-                adamw_elem(x, m, v, load_grad1(p.grad, kBf16, i), a, lam);
-                p.X[i] = x; p.opt_m[i] = m; p.opt_v[i] = v;
+                const uint64_t i = cur.base + e;
+                float xs = p.X[i], ms = p.opt_m[i], vs = p.opt_v[i];
+                adamw_elem(xs, ms, vs, load_grad1(p.grad, kBf16, i), a, cur.lam);
+                p.X[i] = xs; p.opt_m[i] = ms; p.opt_v[i] = vs;
             }
         }
     }
 }
 
-// K3: one SGD-momentum local step on every worker.
+// K3: one SGD-momentum local step on every worker, double-buffered.
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars a) {
     const uint32_t items = p.num_tiles * p.n;
-    for (uint32_t item = blockIdx.x; item < items; item += gridDim.x) {
-        const uint32_t w = item / p.num_tiles;
-        const uint32_t ti = item - w * p.num_tiles;
-        const TileDesc td = p.tiles[ti];
-        const uint64_t base = w * p.d_stride + td.start;
-        const uint32_t e0 = threadIdx.x * kElemsPerThread;
-        if (vector_ok(td, e0)) {
-            float x[8], b[8], g[8];
-            load8(p.X + base + e0, x);
-            load8(p.opt_m + base + e0, b);
-            if (kBf16) load8_bf16(reinterpret_cast<const __nv_bfloat16*>(p.grad) + base + e0, g);
-            else load8(reinterpret_cast<const float*>(p.grad) + base + e0, g);
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+    uint32_t item = blockIdx.x;
+    if (item >= items) return;
+    LocalItem nx = local_item(p, item, e0, false);
+    float x[4], b[4], g[4];
+    if (nx.vec) {
+        load4(p.X + nx.base + e0, x);
+        load4(p.opt_m + nx.base + e0, b);
+        load4_grad<kBf16>(p.grad, nx.base + e0, g);
+    }
+    for (; item < items; item += gridDim.x) {
+        const LocalItem cur = nx;
+        float cx[4], cb[4], cg[4];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) sgdm_elem(x[j], b[j], g[j], a);
-            store8(p.X + base + e0, x);
-            store8(p.opt_m + base + e0, b);
+        for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cb[j] = b[j]; cg[j] = g[j]; }
+        const uint32_t next = item + gridDim.x;
+        if (next < items) {
+            nx = local_item(p, next, e0, false);
+            if (nx.vec) {
+                load4(p.X + nx.base + e0, x);
+                load4(p.opt_m + nx.base + e0, b);
+                load4_grad<kBf16>(p.grad, nx.base + e0, g);
+            }
+        }
+        if (cur.vec) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) sgdm_elem(cx[j], cb[j], cg[j], a);
+            store4(p.X + cur.base + e0, cx);
+            store4(p.opt_m + cur.base + e0, cb);
         } else {
-            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
-                const uint64_t i = base + e;
-                float x = p.X[i], b = p.opt_m[i];
-                sgdm_elem(x, b, load_grad1(p.grad, kBf16, i), a);
-                p.X[i] = x; p.opt_m[i] = b;
+                const uint64_t i = cur.base + e;
+                float xs = p.X[i], bs = p.opt_m[i];
+                sgdm_elem(xs, bs, load_grad1(p.grad, kBf16, i), a);
+                p.X[i] = xs; p.opt_m[i] = bs;
             }
         }
     }
 }
 
+// Global step on one element, any number of workers, reading each replica
+// once for the average and once more for the statistics.
+__device__ __forceinline__ void global_elem_generic(const Problem& p, const GlobalScalars& g, float lam,
+                                                    uint64_t gi, ThreadStats& st) {
+    const float x = p.x[gi], m = p.m[gi];
+    float r = 0.f;
+    if (g.sign_mode != 0) r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
+    float acc = 0.f;
+    for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x, p.X[i * p.d_stride + gi]));
+    const float D = __fdiv_rn(acc, g.n_f);
+    const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
+    const float s = applied_sign(u, g, r);
+    const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
+    const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    const int sD = sgn(D);
+    float dr = 0.f;
+    bool unan = true;
+    for (uint32_t i = 0; i < p.n; ++i) {
+        const float di = __fsub_rn(x, p.X[i * p.d_stride + gi]);
+        const float ei = __fsub_rn(di, D);
+        dr = __fadd_rn(dr, __fmul_rn(ei, ei));
+        unan = unan && (sgn(di) == sD);
+    }
+    csum_add(st.dsq, __fmul_rn(D, D));
+    csum_add(st.drift, dr);
+    st.zero += (s == 0.f);
+    st.flips += (sgn(u) != sD);
+    st.unanimous += unan;
+    st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
+    p.x[gi] = xn;
+    p.m[gi] = mn;
+    for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = xn;
+}
+
 // K4: the fused global step (average over the replicas, sign-momentum update,
-// momentum update, reset of every replica) with per-tile statistics.
-// NW > 0: exactly NW replicas, held in registers.  NW == 0: any n, one
-// element at a time, reading each replica twice.
+// momentum update, reset of every replica) with statistics.
+// NW > 0: exactly NW replicas, held in registers and double-buffered.
+// NW == 0: any n, one element at a time.
+// Statistics: a CTA keeps per-thread sums while its successive tiles belong
+// to one tensor and reduces them only when the tensor changes (or at its last
+// tile), writing the segment's partial at the segment's last tile and zeros
+// at its other tiles; the per-tensor sum over tiles is then unchanged.
 template <int NW>
 __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g) {
-    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
-        const TileDesc td = p.tiles[ti];
-        const float lam = p.tensors[td.tensor].lam_global;
-        const uint32_t e0 = threadIdx.x * kElemsPerThread;
-        ThreadStats st;
-        if (NW > 0 && vector_ok(td, e0)) {
-            constexpr int W = NW > 0 ? NW : 1;
-            const uint64_t gi = td.start + e0;
-            float x[8], m[8], r[W][8];
-            load8(p.x + gi, x);
-            load8(p.m + gi, m);
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+    constexpr int W = NW > 0 ? NW : 1;
+    uint32_t ti = blockIdx.x;
+    if (ti >= p.num_tiles) return;
+    TileDesc nt = p.tiles[ti];
+    bool nvec = NW > 0 && vector_ok(nt, e0);
+    float x[4], m[4], r[W][4];
+    ThreadStats st;
+    if (nvec) {
+        load4(p.x + nt.start + e0, x);
+        load4(p.m + nt.start + e0, m);
 #pragma unroll
-            for (int i = 0; i < W; ++i) load8(p.X + i * p.d_stride + gi, r[i]);
-            float ru[8];
-            if (g.sign_mode != 0) {  // elements gi..gi+7 are the words of two Philox blocks
-                const uint4 b0 = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
-                const uint4 b1 = philox_block((gi >> 2) + 1, g.philox_k0, g.philox_k1);
-                ru[0] = philox_unit(b0.x); ru[1] = philox_unit(b0.y); ru[2] = philox_unit(b0.z); ru[3] = philox_unit(b0.w);
-                ru[4] = philox_unit(b1.x); ru[5] = philox_unit(b1.y); ru[6] = philox_unit(b1.z); ru[7] = philox_unit(b1.w);
-            } else {
+        for (int i = 0; i < W; ++i) load4(p.X + i * p.d_stride + nt.start + e0, r[i]);
+    }
+    for (; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = nt;
+        const bool vec = nvec;
+        float cx[4], cm[4], cr[W][4];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) ru[j] = 0.f;
-            }
+        for (int j = 0; j < 4; ++j) {
+            cx[j] = x[j];
+            cm[j] = m[j];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                float dif[W];
+            for (int i = 0; i < W; ++i) cr[i][j] = r[i][j];
+        }
+        const uint32_t next = ti + gridDim.x;
+        if (next < p.num_tiles) {
+            nt = p.tiles[next];
+            nvec = NW > 0 && vector_ok(nt, e0);
+            if (nvec) {
+                load4(p.x + nt.start + e0, x);
+                load4(p.m + nt.start + e0, m);
 #pragma unroll
-                for (int i = 0; i < W; ++i) dif[i] = __fsub_rn(x[j], r[i][j]);
-                global_elem<W>(x[j], m[j], dif, W, g, lam, ru[j], st);
-            }
-            store8(p.x + gi, x);
-            store8(p.m + gi, m);
-#pragma unroll
-            for (int i = 0; i < W; ++i) store8(p.X + i * p.d_stride + gi, x);
-        } else {
-            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
-            for (uint32_t e = e0; e < e1; ++e) {
-                const uint64_t gi = td.start + e;
-                float x = p.x[gi], m = p.m[gi];
-                float r = 0.f;
-                if (g.sign_mode != 0)
-                    r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
-                // one element, any number of workers: the worker differences are read
-                // once for the average and once more for the statistics
-                float acc = 0.f;
-                for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x, p.X[i * p.d_stride + gi]));
-                const float D = __fdiv_rn(acc, g.n_f);
-                const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
-                const float s = applied_sign(u, g, r);
-                const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
-                const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
-                const int sD = sgn(D);
-                float dr = 0.f;
-                bool unan = true;
-                for (uint32_t i = 0; i < p.n; ++i) {
-                    const float di = __fsub_rn(x, p.X[i * p.d_stride + gi]);
-                    const float ei = __fsub_rn(di, D);
-                    dr = __fadd_rn(dr, __fmul_rn(ei, ei));
-                    unan = unan && (sgn(di) == sD);
-                }
-                st.dsq = __fadd_rn(st.dsq, __fmul_rn(D, D));
-                st.drift = __fadd_rn(st.drift, dr);
-                st.zero += (s == 0.f);
-                st.flips += (sgn(u) != sD);
-                st.unanimous += unan;
-                st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
-                p.x[gi] = xn;
-                p.m[gi] = mn;
-                for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = xn;
+                for (int i = 0; i < W; ++i) load4(p.X + i * p.d_stride + nt.start + e0, r[i]);
             }
         }
-        reduce_stats(st, p.partials + ti);
+        const float lam = p.tensors[td.tensor].lam_global;
+        if (vec) {
+            const uint64_t gi = td.start + e0;  // a multiple of 4: the four words of one Philox block
+            float ru[4] = {0.f, 0.f, 0.f, 0.f};
+            if (g.sign_mode != 0) {
+                const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float dif[W];
+#pragma unroll
+                for (int i = 0; i < W; ++i) dif[i] = __fsub_rn(cx[j], cr[i][j]);
+                global_elem<W>(cx[j], cm[j], dif, W, g, lam, ru[j], st);
+            }
+            store4(p.x + gi, cx);
+            store4(p.m + gi, cm);
+#pragma unroll
+            for (int i = 0; i < W; ++i) store4(p.X + i * p.d_stride + gi, cx);
+        } else {
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) global_elem_generic(p, g, lam, td.start + e, st);
+        }
+        if (next >= p.num_tiles || nt.tensor != td.tensor) {  // uniform across the CTA
+            reduce_stats(st, p.partials + ti);
+            st = ThreadStats();
+        } else {
+            zero_partial(p.partials + ti);
+        }
     }
 }
 

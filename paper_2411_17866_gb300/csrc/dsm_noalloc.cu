@@ -155,7 +155,7 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     }
     if (d == 0) return na_fail(DSM_EINVAL, "the model has no elements");
     if (tiles > kNaMaxTiles)
-        return na_fail(DSM_ERANGE, "layout needs more than DSM_NOALLOC_MAX_TILES (524288) tiles of 2048 elements");
+        return na_fail(DSM_ERANGE, "layout needs more than DSM_NOALLOC_MAX_TILES (524288) tiles of 1024 elements");
     if (replica_stride < d || replica_stride % 8 != 0)
         return na_fail(DSM_EINVAL, "replica_stride must be >= d and a multiple of 8");
     if (!aligned16(x) || !aligned16(m) || !aligned16(replicas))

@@ -125,6 +125,24 @@ def pin_uniform24(o):
     b = o.uniform24(11, 1, 3, e)
     assert np.mean(a == b) < 1e-3          # the two streams are separated
     assert abs(np.corrcoef(a, b)[0, 1]) < 5e-3
+    # the two draws taken from one 64-bit output are uncorrelated
+    assert abs(np.corrcoef(a[0::2], a[1::2])[0, 1]) < 5e-3
+
+
+def pin_hash_fields(o):
+    """Elements 2q and 2q+1 take bits 63..40 and 39..16 of SplitMix64 output q+1 of the family's key."""
+    seed, stream, idx = 7, 1, 5
+    key = np.array([o.hash_key(seed, stream, idx)], dtype=np.uint64)
+    e = np.array([0, 1, 2, 3, 1001], dtype=np.int64)
+    h = o.hash24(seed, stream, idx, e)
+    for ei, hi in zip(e.tolist(), h.tolist()):
+        out = int(o.splitmix64_output(key, np.array([ei // 2 + 1], dtype=np.uint64))[0])
+        want = (out >> 40) & 0xFFFFFF if ei % 2 == 0 else (out >> 16) & 0xFFFFFF
+        assert hi == want, (ei, hi, want)
+    # the family key is output 1 + stream*2^40 + idx of SplitMix64(seed)
+    want_key = int(o.splitmix64_output(np.array([seed], dtype=np.uint64),
+                                       np.array([1 + (stream << 40) + idx], dtype=np.uint64))[0])
+    assert int(key[0]) == want_key
 
 
 def pin_synthetic_grad(o):
@@ -435,7 +453,7 @@ def pin_fp32_vs_fp64(o):
 
 
 PINS = [pin_worked_example, pin_splitmix64, pin_philox, pin_philox_uniform_mapping, pin_bf16,
-        pin_uniform24, pin_synthetic_grad, pin_adamw_vs_torch, pin_adamw_constant_grad,
+        pin_uniform24, pin_hash_fields, pin_synthetic_grad, pin_adamw_vs_torch, pin_adamw_constant_grad,
         pin_adamw_first_step_fp32, pin_sgdm_vs_torch, pin_sgd_plain_exact, pin_sgdm_constant_grad,
         pin_lion, pin_signsgd_momentum, pin_identical_workers, pin_tau1_pseudo_gradient,
         pin_sign_range, pin_lemma1, pin_stats, pin_subset_mode, pin_fp32_vs_fp64]

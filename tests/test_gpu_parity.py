@@ -4,7 +4,7 @@ Tolerance: bit-exact.  The kernels evaluate the oracle's fp32 expression
 trees one rounding at a time (no contraction), with the same worker order,
 so x, m, every replica, every base-optimizer state and every gradient must
 be identical bit for bit.  The statistics' sums are compared to a relative
-1e-5 (see gpu_common.STATS_RTOL); their counts exactly.
+(n + 4) * 2^-24 (derived in gpu_common.stats_rtol); their counts exactly.
 """
 import dataclasses
 
@@ -76,7 +76,7 @@ def test_rounds_bitexact(layout_name, name, hp, n, tau):
         stats = run.global_step(with_stats=True)
         ora.global_step()
         compare_state(run, ora)
-        compare_stats(stats, ora.last_stats)
+        compare_stats(stats, ora.last_stats, n)
     run.close()
 
 
@@ -211,7 +211,7 @@ def test_full_workloads_sampled(key):
         if ora.opt_v is not None:
             assert_bitexact(rd(dsm.BUF_OPT_V, i), ora.opt_v[i], f"opt_v {i}")
     if elems is None:
-        compare_stats(stats, ora.last_stats)
+        compare_stats(stats, ora.last_stats, wl.n)
     else:
         # properties that hold at any size
         assert sum(s["unanimous"] for s in stats) <= wl.d

@@ -60,6 +60,9 @@ MUTANTS = [
      [P.pin_philox_uniform_mapping]),
     ("splitmix_shift", "z = (z ^ (z >> U64(27))) * U64(_MIX_C2)", "z = (z ^ (z >> U64(28))) * U64(_MIX_C2)",
      [P.pin_splitmix64]),
+    ("hash_fields_swapped", "shift = np.where((e & U64(1)) == 0, U64(40), U64(16))",
+     "shift = np.where((e & U64(1)) == 0, U64(16), U64(40))",
+     [P.pin_hash_fields]),
     ("bf16_round_half_up", "r = ((b + U64(0x7FFF) + kept_lsb) >> U64(16)) << U64(16)",
      "r = ((b + U64(0x8000)) >> U64(16)) << U64(16)",
      [P.pin_bf16]),

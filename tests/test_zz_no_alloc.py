@@ -18,7 +18,7 @@ import dataclasses
 import pytest
 
 import workloads as W
-from gpu_common import STATS_RTOL
+from gpu_common import stats_rtol
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -34,12 +34,12 @@ CASES = [("adamw-sign-n4", W.HParams(), 4, 2),
          ("adamw-rsign0-n9", dataclasses.replace(W.HParams(), sign_mode=W.RSIGN_ZERO, rsign_B=1.0), 9, 1)]
 
 
-def _stats_close(a, b):
+def _stats_close(a, b, n):
     for ta, tb in zip(a, b):
         for key in ("zero_sign", "flips", "unanimous", "clamped"):
             assert ta[key] == tb[key], key
         for key in ("delta_sq", "drift"):
-            assert abs(ta[key] - tb[key]) <= STATS_RTOL * abs(tb[key]), key
+            assert abs(ta[key] - tb[key]) <= stats_rtol(n) * abs(tb[key]), key
 
 
 @pytest.mark.parametrize("name,hp,n,tau", CASES, ids=[c[0] for c in CASES])
@@ -75,7 +75,7 @@ def test_noalloc_global_step_matches_handle_path(name, hp, n, tau):
         for i in range(n):
             got = reps[i * stride:i * stride + d].cpu().view(torch.int32)
             assert torch.equal(got, run.read(dsm.BUF_REPLICA, i).view(torch.int32))
-        _stats_close([s.as_dict() for s in host_stats], want_stats)
+        _stats_close([s.as_dict() for s in host_stats], want_stats, n)
         # statistics written to device memory instead
         if call == 1:
             dev_stats = torch.zeros(len(LAYOUT) * 6, dtype=torch.float64, device="cuda")
@@ -91,11 +91,11 @@ def test_noalloc_global_step_matches_handle_path(name, hp, n, tau):
 def test_noalloc_rejects_sizes_beyond_its_limit():
     if not torch.cuda.is_available():
         pytest.skip("no GPU")
-    big = (W.Tensor("huge", (dsm_max_tiles() + 1) * 2048, W.KIND_WEIGHT, 1e-3),)
+    big = (W.Tensor("huge", (dsm_max_tiles() + 1) * 1024, W.KIND_WEIGHT, 1e-3),)
     x = torch.empty(16, dtype=torch.float32, device="cuda")
     with pytest.raises(dsm.DsmError) as e:
         dsm.dsm_global_step_noalloc(dsm.make_layout(big), 2, dsm.make_hparams(W.HParams()), 1e-3, 0,
-                                    x.data_ptr(), x.data_ptr(), x.data_ptr(), (dsm_max_tiles() + 1) * 2048)
+                                    x.data_ptr(), x.data_ptr(), x.data_ptr(), (dsm_max_tiles() + 1) * 1024)
     assert e.value.code == dsm.DSM_ERANGE and "DSM_NOALLOC_MAX_TILES" in str(e.value)
     many = tuple(W.Tensor(f"t{i}", 8, W.KIND_BIAS, 1e-3) for i in range(4097))
     with pytest.raises(dsm.DsmError) as e:
