@@ -92,6 +92,28 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(seconds: float, world: int) -> float:
+    """The slowest rank's time (host-side gloo reduction; nothing on the data path)."""
+    if world <= 1:
+        return seconds
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([seconds], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def shard_hparams(hp, rank: int):
+    """Each rank's parameter shard draws its own synthetic inputs (seed + rank)."""
+    import dataclasses
+    return dataclasses.replace(hp, seed=hp.seed + rank)
+
+
+def whole_job_value(d_per_rank: int, world: int, rounds: int, seconds: float) -> float:
+    """params/s over all ranks: every rank processes its own shard of d parameters per round."""
+    return world * d_per_rank * rounds / seconds
+
+
 def bytes_per_elem_local(wl) -> int:
     """Algorithmic bytes of one local step per worker-element: every state read and written once."""
     g = 2 if wl.hp.grad_dtype == W.BF16 else 4
@@ -252,8 +274,7 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     wl = select_workload(args)
-    import dataclasses
-    hp = dataclasses.replace(wl.hp, seed=wl.hp.seed + rank)
+    hp = shard_hparams(wl.hp, rank)
     run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp, device=dev)
     stream = torch.cuda.current_stream(dev)
     tau = wl.tau
@@ -304,11 +325,7 @@ def main():
     if world > 1:
         dist.barrier()
     clocks = sampler.stop() if sampler else None
-    elapsed = start.elapsed_time(end) / 1e3
-    if world > 1:
-        tt = torch.tensor([elapsed], dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed = float(tt.item())
+    elapsed = max_over_ranks(start.elapsed_time(end) / 1e3, world)
     local_ms = [a.elapsed_time(b) for a, b in local_ev]
     global_ms = [a.elapsed_time(b) for a, b in global_ev]
 
@@ -334,12 +351,8 @@ def main():
             run.global_step(stream)
             run.read(dsm.BUF_X, out=host_x, stream=stream)   # synchronises the stream
             t += 1
-        e2e_dt = time.perf_counter() - t0
-        if world > 1:
-            tt = torch.tensor([e2e_dt], dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_dt = float(tt.item())
-        e2e = {"value": world * wl.d * args.e2e_steps / e2e_dt, "unit": UNIT,
+        e2e_dt = max_over_ranks(time.perf_counter() - t0, world)
+        e2e = {"value": whole_job_value(wl.d, world, args.e2e_steps, e2e_dt), "unit": UNIT,
                "h2d_bytes_per_step": tau * wl.n * wl.d * esz, "d2h_bytes_per_step": wl.d * 4,
                "steps": args.e2e_steps, "path": "dsm_load_grads (pinned host) + dsm_local_step x tau, "
                                                  "dsm_global_step, dsm_read_params(x -> pinned host)"}
@@ -357,7 +370,7 @@ def main():
     traffic = committed_traffic(f"{kname}:{args.workload}")
     global_bytes = wl.d * bytes_per_param_global(wl)
     avg_global_s = statistics.mean(global_ms) / 1e3
-    value = world * wl.d * args.steps / elapsed
+    value = whole_job_value(wl.d, world, args.steps, elapsed)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,

@@ -370,9 +370,13 @@ int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     const size_t es = h->al.grad_esize;
-    cudaError_t err = cudaMemcpy2DAsync(h->prob.grad, h->al.d_stride * es, src, h->al.d * es, h->al.d * es, h->n,
-                                        src_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice,
-                                        S(stream));
+    const cudaMemcpyKind kind = src_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    cudaError_t err;
+    if (h->al.d_stride == h->al.d)  // the workers' slices are contiguous: one linear copy
+        err = cudaMemcpyAsync(h->prob.grad, src, h->al.d * es * h->n, kind, S(stream));
+    else
+        err = cudaMemcpy2DAsync(h->prob.grad, h->al.d_stride * es, src, h->al.d * es, h->al.d * es, h->n, kind,
+                                S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "copy gradients");
     return DSM_OK;
 }

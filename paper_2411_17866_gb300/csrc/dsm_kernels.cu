@@ -332,12 +332,13 @@ __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
         const float s = T.scale, s2 = T.scale2;
         if (vector_ok(td, e0)) {
             const uint64_t gi = td.start + e0;  // even: elements gi..gi+3 use outputs gi/2+1, gi/2+2
-            const uint64_t j = (gi >> 1) + 1;
-            const uint64_t h0 = sm64_output(k.step, j), h1 = sm64_output(k.step, j + 1);
+            // output j of any family is finalise(key + j*gamma): j*gamma is shared by all families
+            const uint64_t jg0 = ((gi >> 1) + 1) * kGoldenGamma, jg1 = jg0 + kGoldenGamma;
+            const uint64_t h0 = sm64_finalise(k.step + jg0), h1 = sm64_finalise(k.step + jg1);
             const float a[4] = {step_term(s, draw_even(h0)), step_term(s, draw_odd(h0)),
                                 step_term(s, draw_even(h1)), step_term(s, draw_odd(h1))};
             for (uint32_t w = 0; w < p.n; ++w) {
-                const uint64_t q0 = sm64_output(k.worker[w], j), q1 = sm64_output(k.worker[w], j + 1);
+                const uint64_t q0 = sm64_finalise(k.worker[w] + jg0), q1 = sm64_finalise(k.worker[w] + jg1);
                 const float g[4] = {grad_value(a[0], s2, draw_even(q0)), grad_value(a[1], s2, draw_odd(q0)),
                                     grad_value(a[2], s2, draw_even(q1)), grad_value(a[3], s2, draw_odd(q1))};
                 const uint64_t o = w * p.d_stride + gi;
