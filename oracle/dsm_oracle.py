@@ -18,6 +18,9 @@ What it computes (arXiv 2411.17866):
   (rand-sign-2), driven by Philox4x32-10.
 * Per-tensor round statistics (squared norm of the averaged pseudo-gradient,
   worker drift, sign counts), accumulated in float64 in element order.
+* The global-step variants of the ablations (Sec. 5): SlowMo (Appendix A,
+  Algorithm "SlowMo"), signed SlowMo and Lookahead (Sec. 5, ablation
+  studies), and the global AdamW step (Appendix, Algorithm "global AdamW").
 
 Precision.  The paper fixes no precision.  Every function is generic in the
 float dtype: ``np.float32`` is the canonical mode whose expression trees the
@@ -298,15 +301,10 @@ def global_step(x, m, X, gamma, b1, b2, eta, lam_e, sign_mode: int, B, r, dt):
     intermediates (Delta, u, the applied sign, the worker differences).
     """
     T = dt.type
-    n = len(X)
     c1 = T((1.0 - f32(b1)) / f32(gamma))
     c2 = T((1.0 - f32(b2)) / f32(gamma))
     eg = T(f32(eta) * f32(gamma))
-    diffs = [x - X[i] for i in range(n)]
-    acc = np.zeros_like(x)
-    for i in range(n):
-        acc = acc + diffs[i]
-    delta = acc / T(n)
+    delta, diffs = worker_average(x, X, dt)
     u = T(f32(b1)) * m + c1 * delta
     if sign_mode == 0:
         sg = sign(u)
@@ -315,6 +313,80 @@ def global_step(x, m, X, gamma, b1, b2, eta, lam_e, sign_mode: int, B, r, dt):
     x_new = x - eg * (sg + lam_e * x)
     m_new = T(f32(b2)) * m + c2 * delta
     return x_new, m_new, {"delta": delta, "u": u, "sg": sg, "diffs": diffs}
+
+
+GLOBAL_SIGN_MOMENTUM = 0   # Algorithm 1
+GLOBAL_SLOWMO = 1          # Appendix A, Algorithm "SlowMo"
+GLOBAL_SIGNED_SLOWMO = 2   # Sec. 5, signed SlowMo
+GLOBAL_LOOKAHEAD = 3       # Sec. 5, Lookahead (Eq. (model-update) replaced)
+GLOBAL_ADAMW = 4           # Appendix, Algorithm "global AdamW"
+
+
+def worker_average(x, X, dt):
+    """Delta = (1/n) sum_i (x - x_i), summed over i = 0..n-1 in order (the all-reduce average)."""
+    n = len(X)
+    diffs = [x - X[i] for i in range(n)]
+    acc = np.zeros_like(x)
+    for i in range(n):
+        acc = acc + diffs[i]
+    return acc / dt.type(n), diffs
+
+
+def global_step_slowmo(x, m, X, gamma, beta, alpha, dt):
+    """SlowMo (Appendix A): exact averaging; u <- beta u + (1/gamma)(x - xbar); x <- x - alpha gamma u.
+
+    ``m`` holds the slow momentum u.  Returns x', u', intermediates.
+    """
+    T = dt.type
+    delta, diffs = worker_average(x, X, dt)
+    inv_g = T(1.0 / f32(gamma))
+    u = T(f32(beta)) * m + inv_g * delta
+    x_new = x - T(f32(alpha) * f32(gamma)) * u
+    return x_new, u, {"delta": delta, "u": u, "sg": sign(u), "diffs": diffs}
+
+
+def global_step_signed_slowmo(x, m, X, gamma, b1, b2, eta, dt):
+    """Signed SlowMo (Sec. 5): u = b1 m + ((1-b1)/gamma) sign(x - xbar); x' = x - eta gamma u;
+    the momentum update, Eq. (mom-update), is kept: m' = b2 m + ((1-b2)/gamma)(x - xbar)."""
+    T = dt.type
+    delta, diffs = worker_average(x, X, dt)
+    c1 = T((1.0 - f32(b1)) / f32(gamma))
+    c2 = T((1.0 - f32(b2)) / f32(gamma))
+    sd = sign(delta)
+    u = T(f32(b1)) * m + c1 * sd
+    x_new = x - T(f32(eta) * f32(gamma)) * u
+    m_new = T(f32(b2)) * m + c2 * delta
+    return x_new, m_new, {"delta": delta, "u": u, "sg": sd, "diffs": diffs}
+
+
+def global_step_lookahead(x, m, X, gamma, b1, b2, eta, dt):
+    """Lookahead (Sec. 5): Algorithm 1 with Eq. (model-update) replaced by x' = x - eta gamma u."""
+    T = dt.type
+    delta, diffs = worker_average(x, X, dt)
+    c1 = T((1.0 - f32(b1)) / f32(gamma))
+    c2 = T((1.0 - f32(b2)) / f32(gamma))
+    u = T(f32(b1)) * m + c1 * delta
+    x_new = x - T(f32(eta) * f32(gamma)) * u
+    m_new = T(f32(b2)) * m + c2 * delta
+    return x_new, m_new, {"delta": delta, "u": u, "sg": sign(u), "diffs": diffs}
+
+
+def global_step_adamw(x, m, v, X, gamma, t: int, b1, b2, eps, eta, lam_e, dt):
+    """Global AdamW with local steps (Appendix, Algorithm "global AdamW") at round t (0-based).
+
+    g = (1/gamma)(x - xbar); m <- b1 m + (1-b1) g; v <- b2 v + (1-b2) g*g;
+    mhat = m/(1 - b1^(t+1)); vhat = v/(1 - b2^(t+1));
+    x' = x - eta (mhat/(sqrt(vhat) + eps) + lam x).
+    """
+    T = dt.type
+    delta, diffs = worker_average(x, X, dt)
+    g = T(1.0 / f32(gamma)) * delta
+    m_new = T(f32(b1)) * m + T(1.0 - f32(b1)) * g
+    v_new = T(f32(b2)) * v + T(1.0 - f32(b2)) * (g * g)
+    mhat = m_new / T(1.0 - beta_power(b1, t + 1))
+    vhat = v_new / T(1.0 - beta_power(b2, t + 1))
+    x_new = x - T(f32(eta)) * (mhat / (np.sqrt(vhat) + T(f32(eps))) + lam_e * x)
+    return x_new, m_new, v_new, {"delta": delta, "u": m_new, "sg": sign(m_new), "diffs": diffs}
 
 
 STAT_FIELDS = ("delta_sq", "drift", "zero_sign", "flips", "unanimous", "clamped")
@@ -406,6 +478,8 @@ class OracleRun:
         self.X = [self.x.copy() for _ in range(self.n)]
         self.opt_m = [np.zeros_like(self.x) for _ in range(self.n)]
         self.opt_v = [np.zeros_like(self.x) for _ in range(self.n)] if hp.base == 0 else None
+        self.global_mode = getattr(hp, "global_mode", GLOBAL_SIGN_MOMENTUM)
+        self.gv = np.zeros_like(self.x) if self.global_mode == GLOBAL_ADAMW else None
         self.t = 0
         self.k = 0
         self.gamma = hp.lr
@@ -435,13 +509,31 @@ class OracleRun:
         """All-reduce average, sign-momentum update and synchronisation (Algorithm 1)."""
         assert self.k == self.tau
         hp = self.hp
-        r = None
-        if hp.sign_mode != 0:
-            r = philox_uniform(self.elems, hp.seed, self.t)
-        x_new, m_new, inter = global_step(self.x, self.m, self.X, self.gamma, hp.g_b1, hp.g_b2,
-                                          hp.g_eta, self.wd_global, hp.sign_mode, hp.rsign_B, r, self.dt)
+        mode = self.global_mode
+        if mode == GLOBAL_SIGN_MOMENTUM:
+            r = None
+            if hp.sign_mode != 0:
+                r = philox_uniform(self.elems, hp.seed, self.t)
+            x_new, m_new, inter = global_step(self.x, self.m, self.X, self.gamma, hp.g_b1, hp.g_b2,
+                                              hp.g_eta, self.wd_global, hp.sign_mode, hp.rsign_B, r, self.dt)
+        elif mode == GLOBAL_SLOWMO:
+            x_new, m_new, inter = global_step_slowmo(self.x, self.m, self.X, self.gamma, hp.g_b1, hp.g_eta,
+                                                     self.dt)
+        elif mode == GLOBAL_SIGNED_SLOWMO:
+            x_new, m_new, inter = global_step_signed_slowmo(self.x, self.m, self.X, self.gamma, hp.g_b1,
+                                                            hp.g_b2, hp.g_eta, self.dt)
+        elif mode == GLOBAL_LOOKAHEAD:
+            x_new, m_new, inter = global_step_lookahead(self.x, self.m, self.X, self.gamma, hp.g_b1, hp.g_b2,
+                                                        hp.g_eta, self.dt)
+        elif mode == GLOBAL_ADAMW:
+            x_new, m_new, self.gv, inter = global_step_adamw(self.x, self.m, self.gv, self.X, self.gamma, self.t,
+                                                             hp.g_b1, hp.g_b2, hp.g_eps, hp.g_eta,
+                                                             self.wd_global, self.dt)
+        else:
+            raise ValueError(f"global mode {mode} unknown")
         if self.with_stats:
-            self.last_stats = round_stats(inter, self.tensor_of, len(self.tensors), hp.sign_mode, hp.rsign_B)
+            self.last_stats = round_stats(inter, self.tensor_of, len(self.tensors),
+                                          hp.sign_mode if mode == GLOBAL_SIGN_MOMENTUM else 0, hp.rsign_B)
         self.last_inter = inter
         self.x, self.m = x_new, m_new
         self.X = [x_new.copy() for _ in range(self.n)]

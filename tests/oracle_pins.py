@@ -452,8 +452,90 @@ def pin_fp32_vs_fp64(o):
             assert np.all(np.abs(a.m - b.m)[ok] <= tol_m)
 
 
+# ---------------------------------------------------------------------------
+# Global-step variants of the ablations (Sec. 5) against textbook special cases
+# ---------------------------------------------------------------------------
+
+def _one_worker_sgd_rounds(o, hp, rounds, rng, d=3000):
+    """n = 1, tau = 1, plain-SGD local step: the pseudo-gradient (x - x_1)/gamma is the gradient itself
+    (up to the rounding of x - gamma g).  Returns the run, the initial model and the gradients used."""
+    x0 = rng.standard_normal(d)
+    run = o.OracleRun(W.flat_layout(d, 1.0), 1, 1, hp, x0=x0, dtype=np.float64)
+    gs = [rng.standard_normal(d).astype(np.float32).astype(np.float64) for _ in range(rounds)]
+    return run, x0, gs
+
+
+def pin_slowmo_heavy_ball(o):
+    """SlowMo with one worker and one plain-SGD step is heavy-ball momentum on g with lr alpha*gamma
+    (torch.optim.SGD(momentum=beta))."""
+    import torch
+    rng = np.random.default_rng(12)
+    gamma, beta, alpha = 2.0 ** -4, 0.7, 0.5
+    hp = W.HParams(base=W.BASE_SGDM, lr=gamma, mu=0.0, g_b1=beta, g_eta=alpha, global_mode=W.GLOBAL_SLOWMO)
+    run, x0, gs = _one_worker_sgd_rounds(o, hp, 5, rng)
+    p = torch.tensor(x0.copy(), dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.SGD([p], lr=o.f32(alpha) * o.f32(gamma), momentum=o.f32(beta), dampening=0.0, foreach=False)
+    for g in gs:
+        run.run_round([[g]])
+        p.grad = torch.tensor(g)
+        opt.step()
+        assert np.allclose(run.x, p.detach().numpy(), rtol=1e-12, atol=1e-13)
+
+
+def pin_lookahead_slow_weights(o):
+    """Lookahead with beta1 = beta2 = 0 is Zhang et al.'s slow-weight update x' = x + eta (xbar - x);
+    with eta = 1 it is plain model averaging (local SGD)."""
+    rng = np.random.default_rng(13)
+    d, n = 2000, 3
+    for eta in (0.5, 1.0):
+        hp = W.HParams(base=W.BASE_SGDM, lr=2.0 ** -5, mu=0.0, g_b1=0.0, g_b2=0.0, g_eta=eta,
+                       global_mode=W.GLOBAL_LOOKAHEAD)
+        run = o.OracleRun(W.flat_layout(d, 1.0), n, 2, hp, x0=rng.standard_normal(d), dtype=np.float64)
+        for _ in range(2):
+            for k in range(2):
+                run.local_step([rng.standard_normal(d).astype(np.float32) for _ in range(n)])
+            xbar = np.mean(np.stack(run.X), axis=0)
+            x = run.x.copy()
+            run.global_step()
+            assert np.allclose(run.x, x + o.f32(eta) * (xbar - x), rtol=1e-12, atol=1e-14)
+
+
+def pin_signed_slowmo_signsgd(o):
+    """Signed SlowMo with beta1 = 0 is signSGD on the averaged pseudo-gradient: x' = x - eta sign(x - xbar)."""
+    rng = np.random.default_rng(14)
+    d, n = 2000, 2
+    hp = W.HParams(base=W.BASE_SGDM, lr=2.0 ** -5, mu=0.0, g_b1=0.0, g_b2=0.9, g_eta=0.25,
+                   global_mode=W.GLOBAL_SIGNED_SLOWMO)
+    run = o.OracleRun(W.flat_layout(d, 1.0), n, 1, hp, x0=rng.standard_normal(d), dtype=np.float64)
+    for _ in range(3):
+        run.local_step([rng.standard_normal(d).astype(np.float32) for _ in range(n)])
+        xbar = np.mean(np.stack(run.X), axis=0)
+        x = run.x.copy()
+        run.global_step()
+        assert np.allclose(run.x, x - 0.25 * np.sign(x - xbar), rtol=1e-14, atol=1e-14)
+
+
+def pin_global_adamw_vs_torch(o):
+    """Global AdamW with one worker and one plain-SGD step is AdamW on g with lr eta (torch.optim.AdamW)."""
+    import torch
+    rng = np.random.default_rng(15)
+    gamma, eta = 2.0 ** -4, 1e-2
+    hp = W.HParams(base=W.BASE_SGDM, lr=gamma, mu=0.0, g_b1=0.9, g_b2=0.95, g_eps=1e-8, g_eta=eta, g_wd=0.1,
+                   global_mode=W.GLOBAL_ADAMW)
+    run, x0, gs = _one_worker_sgd_rounds(o, hp, 6, rng)
+    p = torch.tensor(x0.copy(), dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.AdamW([p], lr=o.f32(eta), betas=(o.f32(0.9), o.f32(0.95)), eps=o.f32(1e-8),
+                            weight_decay=o.f32(0.1), foreach=False)
+    for g in gs:
+        run.run_round([[g]])
+        p.grad = torch.tensor(g)
+        opt.step()
+        assert np.allclose(run.x, p.detach().numpy(), rtol=1e-10, atol=1e-12)
+
+
 PINS = [pin_worked_example, pin_splitmix64, pin_philox, pin_philox_uniform_mapping, pin_bf16,
         pin_uniform24, pin_hash_fields, pin_synthetic_grad, pin_adamw_vs_torch, pin_adamw_constant_grad,
         pin_adamw_first_step_fp32, pin_sgdm_vs_torch, pin_sgd_plain_exact, pin_sgdm_constant_grad,
         pin_lion, pin_signsgd_momentum, pin_identical_workers, pin_tau1_pseudo_gradient,
-        pin_sign_range, pin_lemma1, pin_stats, pin_subset_mode, pin_fp32_vs_fp64]
+        pin_sign_range, pin_lemma1, pin_stats, pin_subset_mode, pin_fp32_vs_fp64,
+        pin_slowmo_heavy_ball, pin_lookahead_slow_weights, pin_signed_slowmo_signsgd, pin_global_adamw_vs_torch]

@@ -17,17 +17,20 @@ SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), 
 
 # (id, original text, planted mistake, pins expected to catch it)
 MUTANTS = [
-    ("global_beta_swapped", "u = T(f32(b1)) * m + c1 * delta", "u = T(f32(b2)) * m + c1 * delta",
+    ("global_beta_swapped", "u = T(f32(b1)) * m + c1 * delta\n    if sign_mode == 0:",
+     "u = T(f32(b2)) * m + c1 * delta\n    if sign_mode == 0:",
      [P.pin_worked_example]),
-    ("global_no_inv_gamma", "c1 = T((1.0 - f32(b1)) / f32(gamma))", "c1 = T((1.0 - f32(b1)))",
+    ("global_no_inv_gamma", "c1 = T((1.0 - f32(b1)) / f32(gamma))\n    c2 = T((1.0 - f32(b2)) / f32(gamma))\n    eg",
+     "c1 = T((1.0 - f32(b1)))\n    c2 = T((1.0 - f32(b2)) / f32(gamma))\n    eg",
      [P.pin_worked_example]),
-    ("global_mom_coeff", "m_new = T(f32(b2)) * m + c2 * delta", "m_new = T(f32(b2)) * m + c1 * delta",
+    ("global_mom_coeff", "    m_new = T(f32(b2)) * m + c2 * delta\n    return x_new, m_new, {\"delta\": delta, \"u\": u, \"sg\": sg,",
+     "    m_new = T(f32(b2)) * m + c1 * delta\n    return x_new, m_new, {\"delta\": delta, \"u\": u, \"sg\": sg,",
      [P.pin_worked_example]),
     ("global_no_weight_decay", "x_new = x - eg * (sg + lam_e * x)", "x_new = x - eg * sg",
      [P.pin_worked_example]),
     ("global_diff_sign", "diffs = [x - X[i] for i in range(n)]", "diffs = [X[i] - x for i in range(n)]",
      [P.pin_worked_example]),
-    ("global_mean_divisor", "delta = acc / T(n)", "delta = acc / T(n + 1)",
+    ("global_mean_divisor", "return acc / dt.type(n), diffs", "return acc / dt.type(n + 1), diffs",
      [P.pin_worked_example]),
     ("global_eta_gamma", "eg = T(f32(eta) * f32(gamma))", "eg = T(f32(eta))",
      [P.pin_worked_example]),
@@ -74,6 +77,17 @@ MUTANTS = [
     ("stats_clamp_threshold", "clamp_e = (np.abs(u) > np.asarray(f32(B), dtype=u.dtype))",
      "clamp_e = (np.abs(u) > np.asarray(f32(B) / 2, dtype=u.dtype))",
      [P.pin_stats]),
+    ("slowmo_no_inv_gamma", "u = T(f32(beta)) * m + inv_g * delta", "u = T(f32(beta)) * m + delta",
+     [P.pin_slowmo_heavy_ball]),
+    ("lookahead_signed", "    u = T(f32(b1)) * m + c1 * delta\n    x_new = x - T(f32(eta) * f32(gamma)) * u\n",
+     "    u = T(f32(b1)) * m + c1 * delta\n    x_new = x - T(f32(eta) * f32(gamma)) * sign(u)\n",
+     [P.pin_lookahead_slow_weights]),
+    ("signed_slowmo_unsigned", "u = T(f32(b1)) * m + c1 * sd", "u = T(f32(b1)) * m + c1 * delta",
+     [P.pin_signed_slowmo_signsgd]),
+    ("global_adamw_bias", "mhat = m_new / T(1.0 - beta_power(b1, t + 1))", "mhat = m_new / T(1.0 - beta_power(b1, t + 2))",
+     [P.pin_global_adamw_vs_torch]),
+    ("global_adamw_no_inv_gamma", "g = T(1.0 / f32(gamma)) * delta", "g = delta",
+     [P.pin_global_adamw_vs_torch]),
     ("subset_tensor_lookup", "self.tensor_of = np.searchsorted(self.starts, self.elems, side=\"right\") - 1",
      "self.tensor_of = np.searchsorted(self.starts, self.elems, side=\"left\") - 1",
      [P.pin_subset_mode, P.pin_stats]),

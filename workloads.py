@@ -35,6 +35,12 @@ RSIGN_ZERO = 1    # randomized sign, Eq. (rand-sign-2): 0 or sign(v)
 RSIGN_PM = 2      # randomized sign, Eq. (rand-sign-1): -sign(v) or sign(v)
 F32 = 0
 BF16 = 1
+# Global steps: Algorithm 1 and the variants of the ablations (Sec. 5)
+GLOBAL_SIGN_MOMENTUM = 0
+GLOBAL_SLOWMO = 1
+GLOBAL_SIGNED_SLOWMO = 2
+GLOBAL_LOOKAHEAD = 3
+GLOBAL_ADAMW = 4
 
 VOCAB = 50257
 CONTEXT = 1024
@@ -66,6 +72,8 @@ class HParams:
     rsign_B: float = 1e-2     # bound B of Eqs. (rand-sign-1/2)
     grad_dtype: int = F32
     seed: int = 0
+    global_mode: int = 0      # GLOBAL_* below
+    g_eps: float = 1e-8       # epsilon of the global AdamW step
 
 
 @dataclasses.dataclass(frozen=True)
