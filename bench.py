@@ -56,7 +56,14 @@ def parse():
     ap.add_argument("--n-workers", type=int, default=None)
     ap.add_argument("--tau", type=int, default=None)
     ap.add_argument("--max-params", type=int, default=None)
+    # the global step: Algorithm 1 (default) or a variant of the ablations
+    ap.add_argument("--global-mode", default=None, choices=sorted(GLOBAL_MODES))
     return ap.parse_args()
+
+
+GLOBAL_MODES = {"sign_momentum": W.GLOBAL_SIGN_MOMENTUM, "slowmo": W.GLOBAL_SLOWMO,
+                "signed_slowmo": W.GLOBAL_SIGNED_SLOWMO, "lookahead": W.GLOBAL_LOOKAHEAD,
+                "adamw": W.GLOBAL_ADAMW}
 
 
 def select_workload(args):
@@ -70,6 +77,11 @@ def select_workload(args):
     if args.tau:
         changes["tau"] = args.tau
         notes.append(f"tau={args.tau}")
+    if args.global_mode and GLOBAL_MODES[args.global_mode] != wl.hp.global_mode:
+        mode = GLOBAL_MODES[args.global_mode]
+        changes["hp"] = dataclasses.replace(wl.hp, global_mode=mode,
+                                            sign_mode=wl.hp.sign_mode if mode == W.GLOBAL_SIGN_MOMENTUM else W.SIGN)
+        notes.append(f"global step {args.global_mode}")
     if args.max_params:
         keep, total = [], 0
         for t in wl.tensors:
@@ -78,9 +90,9 @@ def select_workload(args):
             keep.append(t)
             total += t.numel
         changes["tensors"] = tuple(keep)
-        notes.append(f"first {len(keep)} tensors ({total} params)")
+        notes.append(f"reduced to the first {len(keep)} tensors ({total} params)")
     if changes:
-        changes["name"] = wl.name + " [reduced: " + ", ".join(notes) + "]"
+        changes["name"] = wl.name + " [" + ", ".join(notes) + "]"
         wl = dataclasses.replace(wl, **changes)
     return wl
 
@@ -123,7 +135,8 @@ def bytes_per_elem_local(wl) -> int:
 
 
 def bytes_per_param_global(wl) -> int:
-    return 8 * (wl.n + 2)     # read x, m and n replicas; write x, m and n replicas
+    # read x, m (and the global AdamW second moment) and n replicas; write them all
+    return 8 * (wl.n + 2 + (1 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0))
 
 
 def measured_peaks():
@@ -254,6 +267,7 @@ def workload_config(wl, gpus):
             "base": "adamw" if wl.hp.base == W.BASE_ADAMW else "sgd-momentum",
             "grad_dtype": "bf16" if wl.hp.grad_dtype == W.BF16 else "f32",
             "sign": ["sign", "rand-sign-2", "rand-sign-1"][wl.hp.sign_mode],
+            "global_step": {v: k for k, v in GLOBAL_MODES.items()}[wl.hp.global_mode],
             "parallelism": f"param-shard x{gpus}" if gpus > 1 else "single GPU",
             "l2": "inputs larger than L2 (129 MB): each local-step launch streams "
                   f"{wl.n * wl.d * bytes_per_elem_local(wl) / 1e9:.1f} GB"}

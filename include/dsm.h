@@ -77,6 +77,23 @@ extern "C" {
 #define DSM_F32  0
 #define DSM_BF16 1
 
+/* Global step.  Algorithm 1 (the default) or a variant of the ablations
+ * (Sec. 5), all with the same all-reduce average and reset:
+ *   SIGN_MOMENTUM  Eqs. (ut-update), (model-update), (mom-update)
+ *   SLOWMO         Appendix A, Algorithm "SlowMo": u <- b1 u + (1/gamma) Delta (kept in m),
+ *                  x' = x - eta gamma u (eta plays the role of SlowMo's alpha)
+ *   SIGNED_SLOWMO  Sec. 5: u = b1 m + ((1-b1)/gamma) sign(Delta), x' = x - eta gamma u,
+ *                  m' = b2 m + ((1-b2)/gamma) Delta
+ *   LOOKAHEAD      Sec. 5: Algorithm 1 with x' = x - eta gamma u
+ *   ADAMW          Appendix, Algorithm "global AdamW": g = Delta/gamma, AdamW moments m, v with
+ *                  bias corrections 1 - b^(t+1), x' = x - eta (mhat/(sqrt(vhat)+g_eps) + lambda x)
+ * The randomized sign modes apply to SIGN_MOMENTUM only. */
+#define DSM_GLOBAL_SIGN_MOMENTUM 0
+#define DSM_GLOBAL_SLOWMO        1
+#define DSM_GLOBAL_SIGNED_SLOWMO 2
+#define DSM_GLOBAL_LOOKAHEAD     3
+#define DSM_GLOBAL_ADAMW         4
+
 /* Buffers for dsm_read_params / dsm_write_params. */
 #define DSM_BUF_X        0  /* global model x_{t,0} (fp32, d) */
 #define DSM_BUF_M        1  /* global momentum m_t (fp32, d) */
@@ -84,6 +101,7 @@ extern "C" {
 #define DSM_BUF_OPT_M    3  /* worker AdamW first moment, or SGD-momentum buffer (fp32, d) */
 #define DSM_BUF_OPT_V    4  /* worker AdamW second moment (fp32, d); AdamW only */
 #define DSM_BUF_GRAD     5  /* worker gradient buffer (fp32 or bf16 per grad_dtype, d) */
+#define DSM_BUF_GLOBAL_V 6  /* global AdamW second moment (fp32, d); DSM_GLOBAL_ADAMW only */
 
 typedef void* dsm_stream_t;  /* a cudaStream_t */
 
@@ -111,7 +129,7 @@ typedef struct {
     float eps;           /* AdamW epsilon, > 0 (the paper uses 1e-8) */
     float wd;            /* AdamW decoupled weight decay, >= 0 */
     float mu;            /* SGD-momentum coefficient, in [0, 1) */
-    float g_b1, g_b2;    /* global beta1, beta2 of Eqs. (ut-update), (mom-update), in [0, 1] */
+    float g_b1, g_b2;    /* global beta1, beta2 of Eqs. (ut-update), (mom-update), in [0, 1] ([0, 1) for ADAMW) */
     float g_eta;         /* global learning rate eta of Eq. (model-update), >= 0 */
     float g_wd;          /* global decoupled weight decay lambda, >= 0 */
     int32_t sign_mode;   /* DSM_SIGN | DSM_RSIGN_ZERO | DSM_RSIGN_PM */
@@ -119,13 +137,16 @@ typedef struct {
     int32_t grad_dtype;  /* DSM_F32 | DSM_BF16 */
     uint32_t reserved;   /* must be 0 */
     uint64_t seed;       /* seed of the synthetic generators and of the Philox key */
+    int32_t global_mode; /* DSM_GLOBAL_* */
+    float g_eps;         /* epsilon of the global AdamW step, > 0 when global_mode is DSM_GLOBAL_ADAMW */
 } dsm_hparams;
 
 /* Statistics of one global step for one tensor (Algorithm 1's quantities):
  *   delta_sq  = sum_e Delta_e^2, Delta = (1/n) sum_i (x - x_i)      (pseudo-gradient norm, times gamma^2)
  *   drift     = sum_e sum_i ((x_e - x_{i,e}) - Delta_e)^2           (spread of the workers around their mean)
- *   zero_sign = #{e : applied sign = 0}
- *   flips     = #{e : sign(u_e) != sign(Delta_e)}                    (momentum overrides the round's direction)
+ *   zero_sign = #{e : applied sign = 0}  (for the unsigned variants: sign(u) = 0; signed SlowMo: sign(Delta) = 0)
+ *   flips     = #{e : sign(u_e) != sign(Delta_e)}                    (momentum overrides the round's direction;
+ *               u is the new momentum for SlowMo and the new first moment for global AdamW)
  *   unanimous = #{e : sign(x_e - x_{i,e}) = sign(Delta_e) for every worker i}
  *   clamped   = #{e : |u_e| > B} in the randomized modes, else 0
  * Per element the terms are fp32 values; they are summed with compensated

@@ -62,7 +62,7 @@ bool finite(float v) { return std::isfinite(v); }
 struct ArenaLayout {
     uint64_t d = 0, d_stride = 0;
     uint32_t num_tensors = 0, num_tiles = 0;
-    uint64_t off_tensors = 0, off_tiles = 0, off_x = 0, off_m = 0, off_X = 0, off_om = 0, off_ov = 0,
+    uint64_t off_tensors = 0, off_tiles = 0, off_x = 0, off_m = 0, off_gv = 0, off_X = 0, off_om = 0, off_ov = 0,
              off_grad = 0, off_partials = 0, off_stats = 0, total = 0;
     size_t grad_esize = 4;
 };
@@ -89,6 +89,14 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
     if (!(finite(hp->g_wd) && hp->g_wd >= 0.f)) return fail(DSM_EINVAL, "global lambda must be finite and >= 0");
     if (hp->sign_mode != DSM_SIGN && hp->sign_mode != DSM_RSIGN_ZERO && hp->sign_mode != DSM_RSIGN_PM)
         return fail(DSM_EINVAL, "sign mode %d unknown", hp->sign_mode);
+    if (hp->global_mode < DSM_GLOBAL_SIGN_MOMENTUM || hp->global_mode > DSM_GLOBAL_ADAMW)
+        return fail(DSM_EINVAL, "global mode %d unknown", hp->global_mode);
+    if (hp->global_mode != DSM_GLOBAL_SIGN_MOMENTUM && hp->sign_mode != DSM_SIGN)
+        return fail(DSM_EINVAL, "the randomized sign applies to the sign-momentum global step only");
+    if (hp->global_mode == DSM_GLOBAL_ADAMW) {
+        if (!(hp->g_b1 < 1.f) || !(hp->g_b2 < 1.f)) return fail(DSM_EINVAL, "global AdamW betas must lie in [0, 1)");
+        if (!(finite(hp->g_eps) && hp->g_eps > 0.f)) return fail(DSM_EINVAL, "global AdamW eps must be finite and > 0");
+    }
     if (hp->sign_mode != DSM_SIGN && !(finite(hp->rsign_B) && hp->rsign_B > 0.f))
         return fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
     if (hp->grad_dtype != DSM_F32 && hp->grad_dtype != DSM_BF16)
@@ -125,6 +133,7 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
     a.off_tiles = take(uint64_t(a.num_tiles) * sizeof(TileDesc));
     a.off_x = take(a.d_stride * 4);
     a.off_m = take(a.d_stride * 4);
+    a.off_gv = hp->global_mode == DSM_GLOBAL_ADAMW ? take(a.d_stride * 4) : 0;
     a.off_X = take(uint64_t(n) * a.d_stride * 4);
     a.off_om = take(uint64_t(n) * a.d_stride * 4);
     a.off_ov = hp->base == DSM_BASE_ADAMW ? take(uint64_t(n) * a.d_stride * 4) : 0;
@@ -169,6 +178,8 @@ struct dsm_handle {
     float gamma = 0.f;     // gamma_t of this round
     double b1_pow = 1.0;   // beta1^j and beta2^j for the last local step count j
     double b2_pow = 1.0;
+    double gb1_pow = 1.0;  // global AdamW: beta1^t and beta2^t after t global steps
+    double gb2_pow = 1.0;
     uint64_t j = 0;        // local steps done since the start (AdamW step count)
 };
 
@@ -184,6 +195,7 @@ float* buffer_ptr(dsm_handle* h, int which, uint32_t worker) {
         case DSM_BUF_REPLICA: return h->prob.X + ws;
         case DSM_BUF_OPT_M: return h->prob.opt_m + ws;
         case DSM_BUF_OPT_V: return h->prob.opt_v ? h->prob.opt_v + ws : nullptr;
+        case DSM_BUF_GLOBAL_V: return h->prob.gv;
         default: return nullptr;
     }
 }
@@ -191,8 +203,8 @@ float* buffer_ptr(dsm_handle* h, int which, uint32_t worker) {
 // Resolves (which, worker) to a device address and element size.
 int resolve_buffer(dsm_handle* h, int which, uint32_t worker, uint64_t offset, uint64_t count, char** ptr,
                    size_t* esize) {
-    if (which < DSM_BUF_X || which > DSM_BUF_GRAD) return fail(DSM_EINVAL, "buffer %d unknown", which);
-    const bool per_worker = which >= DSM_BUF_REPLICA;
+    if (which < DSM_BUF_X || which > DSM_BUF_GLOBAL_V) return fail(DSM_EINVAL, "buffer %d unknown", which);
+    const bool per_worker = which >= DSM_BUF_REPLICA && which <= DSM_BUF_GRAD;
     if (per_worker && worker >= h->n) return fail(DSM_ERANGE, "worker %u >= n = %u", worker, h->n);
     if (offset > h->al.d || count > h->al.d - offset)
         return fail(DSM_ERANGE, "elements [%llu, %llu) outside the model of %llu", (unsigned long long)offset,
@@ -297,6 +309,8 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     p.d_stride = al.d_stride;
     p.x = reinterpret_cast<float*>(A + al.off_x);
     p.m = reinterpret_cast<float*>(A + al.off_m);
+    p.gv = hp->global_mode == DSM_GLOBAL_ADAMW ? reinterpret_cast<float*>(A + al.off_gv) : nullptr;
+    p.global_mode = hp->global_mode;
     p.X = reinterpret_cast<float*>(A + al.off_X);
     p.opt_m = reinterpret_cast<float*>(A + al.off_om);
     p.opt_v = hp->base == DSM_BASE_ADAMW ? reinterpret_cast<float*>(A + al.off_ov) : nullptr;
@@ -426,12 +440,22 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
         return fail(DSM_EINVAL, "stats holds %u entries, the layout has %u tensors", stats_count, h->al.num_tensors);
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
-    GlobalScalars g;
+    GlobalScalars g{};
     g.b1 = h->hp.g_b1;
     g.b2 = h->hp.g_b2;
     g.c1 = float((1.0 - double(h->hp.g_b1)) / double(h->gamma));
     g.c2 = float((1.0 - double(h->hp.g_b2)) / double(h->gamma));
     g.eta_gamma = float(double(h->hp.g_eta) * double(h->gamma));
+    g.inv_gamma = float(1.0 / double(h->gamma));
+    // global AdamW at step count t+1: beta^(t+1) by successive float64 products
+    const double ngb1 = h->gb1_pow * double(h->hp.g_b1);
+    const double ngb2 = h->gb2_pow * double(h->hp.g_b2);
+    g.omb1 = float(1.0 - double(h->hp.g_b1));
+    g.omb2 = float(1.0 - double(h->hp.g_b2));
+    g.bc1 = float(1.0 - ngb1);
+    g.bc2 = float(1.0 - ngb2);
+    g.eps = h->hp.g_eps;
+    g.eta = h->hp.g_eta;
     g.B = h->hp.rsign_B;
     g.n_f = float(h->n);
     g.sign_mode = h->hp.sign_mode;
@@ -444,6 +468,8 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     if (err != cudaSuccess) return cuda_fail(err, "launch statistics");
     h->t += 1;
     h->k = 0;
+    h->gb1_pow = ngb1;
+    h->gb2_pow = ngb2;
     if (stats) {
         err = cudaMemcpyAsync(stats, h->prob.stats, size_t(h->al.num_tensors) * sizeof(TensorStats),
                               cudaMemcpyDeviceToHost, s);
@@ -510,6 +536,13 @@ int dsm_set_round(dsm_handle* h, uint64_t round) {
     }
     h->b1_pow = p1;
     h->b2_pow = p2;
+    double q1 = 1.0, q2 = 1.0;
+    for (uint64_t i = 0; i < round; ++i) {
+        q1 *= double(h->hp.g_b1);
+        q2 *= double(h->hp.g_b2);
+    }
+    h->gb1_pow = q1;
+    h->gb2_pow = q2;
     return DSM_OK;
 }
 

@@ -68,6 +68,8 @@ struct Problem {
     uint64_t d_stride;     // elements between workers
     float* x;              // [d]
     float* m;              // [d]
+    float* gv;             // [d] global AdamW second moment (global mode 4 only)
+    int global_mode;
     float* X;              // [n][d_stride] replicas
     float* opt_m;          // [n][d_stride]
     float* opt_v;          // [n][d_stride] (AdamW only)
@@ -90,9 +92,13 @@ struct SgdmScalars {
 };
 
 struct GlobalScalars {
-    float b1, b2;          // global betas
+    float b1, b2;          // global betas (SlowMo: b1 is its beta)
     float c1, c2;          // (1 - beta1)/gamma, (1 - beta2)/gamma
     float eta_gamma;       // eta * gamma
+    float inv_gamma;       // 1/gamma (SlowMo, global AdamW)
+    float omb1, omb2;      // global AdamW: 1 - beta1, 1 - beta2
+    float bc1, bc2;        // global AdamW: 1 - beta1^(t+1), 1 - beta2^(t+1)
+    float eps, eta;        // global AdamW epsilon and learning rate
     float B;               // randomized-sign bound
     float n_f;             // n as float (divisor of the average)
     int sign_mode;

@@ -203,21 +203,58 @@ struct ThreadStats {
     uint32_t zero = 0, flips = 0, unanimous = 0, clamped = 0;
 };
 
-// Global step on one element given x, m and the worker differences d_i = x - x_i:
-// Delta = (sum_i d_i)/n; u = b1 m + c1 Delta; x' = x - eta*gamma (S(u) + lam x);
-// m' = b2 m + c2 Delta.  Accumulates the statistics of the element.
-template <int NW>
-__device__ __forceinline__ void global_elem(float& x, float& m, const float (&dif)[NW], int nw,
+// Global-step update of one element from Delta (mode = DSM_GLOBAL_*); returns u
+// and the sign entering the statistics, and updates x, m (and v for AdamW).
+template <int MODE>
+__device__ __forceinline__ void global_update(float D, float& x, float& m, float& v, const GlobalScalars& g,
+                                              float lam, float r, float& u, float& s) {
+    if (MODE == 0) {         // Algorithm 1: Eqs. (ut-update), (model-update), (mom-update)
+        u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
+        s = applied_sign(u, g, r);
+        const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
+        m = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+        x = xn;
+    } else if (MODE == 1) {  // SlowMo: u <- b u + (1/gamma) Delta; x <- x - alpha gamma u
+        u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.inv_gamma, D));
+        s = static_cast<float>(sgn(u));
+        x = __fsub_rn(x, __fmul_rn(g.eta_gamma, u));
+        m = u;
+    } else if (MODE == 2) {  // signed SlowMo: the pseudo-gradient's sign enters u
+        const float sd = static_cast<float>(sgn(D));
+        u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, sd));
+        s = sd;
+        x = __fsub_rn(x, __fmul_rn(g.eta_gamma, u));
+        m = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    } else if (MODE == 3) {  // Lookahead: Algorithm 1 with x' = x - eta gamma u
+        u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
+        s = static_cast<float>(sgn(u));
+        x = __fsub_rn(x, __fmul_rn(g.eta_gamma, u));
+        m = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    } else {                 // global AdamW on the pseudo-gradient Delta/gamma
+        const float gg = __fmul_rn(g.inv_gamma, D);
+        m = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.omb1, gg));
+        v = __fadd_rn(__fmul_rn(g.b2, v), __fmul_rn(g.omb2, __fmul_rn(gg, gg)));
+        const float mhat = __fdiv_rn(m, g.bc1);
+        const float vhat = __fdiv_rn(v, g.bc2);
+        const float den = __fadd_rn(__fsqrt_rn(vhat), g.eps);
+        x = __fsub_rn(x, __fmul_rn(g.eta, __fadd_rn(__fdiv_rn(mhat, den), __fmul_rn(lam, x))));
+        u = m;
+        s = static_cast<float>(sgn(u));
+    }
+}
+
+// Global step on one element given x, m (v) and the worker differences d_i = x - x_i:
+// Delta = (sum_i d_i)/n, then the mode's update.  Accumulates the element's statistics.
+template <int NW, int MODE>
+__device__ __forceinline__ void global_elem(float& x, float& m, float& v, const float (&dif)[NW], int nw,
                                             const GlobalScalars& g, float lam, float r, ThreadStats& st) {
     float acc = 0.f;
 #pragma unroll
     for (int i = 0; i < NW; ++i)
         if (i < nw) acc = __fadd_rn(acc, dif[i]);
     const float D = __fdiv_rn(acc, g.n_f);
-    const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
-    const float s = applied_sign(u, g, r);
-    const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
-    const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    float u, s;
+    global_update<MODE>(D, x, m, v, g, lam, r, u, s);
     // statistics
     const int sD = sgn(D);
     csum_add(st.dsq, __fmul_rn(D, D));
@@ -235,9 +272,7 @@ __device__ __forceinline__ void global_elem(float& x, float& m, const float (&di
     st.zero += (s == 0.f);
     st.flips += (sgn(u) != sD);
     st.unanimous += unan;
-    st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
-    x = xn;
-    m = mn;
+    st.clamped += (MODE == 0 && g.sign_mode != 0 && fabsf(u) > g.B);
 }
 
 // Fixed-order CTA reduction of the per-thread statistics into one partial:
@@ -476,23 +511,24 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
 
 // Global step on one element, any number of workers, reading each replica
 // once for the average and once more for the statistics.
+template <int MODE>
 __device__ __forceinline__ void global_elem_generic(const Problem& p, const GlobalScalars& g, float lam,
                                                     uint64_t gi, ThreadStats& st) {
-    const float x = p.x[gi], m = p.m[gi];
+    float x = p.x[gi], m = p.m[gi], v = MODE == 4 ? p.gv[gi] : 0.f;
+    const float x0 = x;
     float r = 0.f;
-    if (g.sign_mode != 0) r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
+    if (MODE == 0 && g.sign_mode != 0)
+        r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
     float acc = 0.f;
-    for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x, p.X[i * p.d_stride + gi]));
+    for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x0, p.X[i * p.d_stride + gi]));
     const float D = __fdiv_rn(acc, g.n_f);
-    const float u = __fadd_rn(__fmul_rn(g.b1, m), __fmul_rn(g.c1, D));
-    const float s = applied_sign(u, g, r);
-    const float xn = __fsub_rn(x, __fmul_rn(g.eta_gamma, __fadd_rn(s, __fmul_rn(lam, x))));
-    const float mn = __fadd_rn(__fmul_rn(g.b2, m), __fmul_rn(g.c2, D));
+    float u, s;
+    global_update<MODE>(D, x, m, v, g, lam, r, u, s);
     const int sD = sgn(D);
     float dr = 0.f;
     bool unan = true;
     for (uint32_t i = 0; i < p.n; ++i) {
-        const float di = __fsub_rn(x, p.X[i * p.d_stride + gi]);
+        const float di = __fsub_rn(x0, p.X[i * p.d_stride + gi]);
         const float ei = __fsub_rn(di, D);
         dr = __fadd_rn(dr, __fmul_rn(ei, ei));
         unan = unan && (sgn(di) == sD);
@@ -502,10 +538,11 @@ __device__ __forceinline__ void global_elem_generic(const Problem& p, const Glob
     st.zero += (s == 0.f);
     st.flips += (sgn(u) != sD);
     st.unanimous += unan;
-    st.clamped += (g.sign_mode != 0 && fabsf(u) > g.B);
-    p.x[gi] = xn;
-    p.m[gi] = mn;
-    for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = xn;
+    st.clamped += (MODE == 0 && g.sign_mode != 0 && fabsf(u) > g.B);
+    p.x[gi] = x;
+    p.m[gi] = m;
+    if (MODE == 4) p.gv[gi] = v;
+    for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = x;
 }
 
 // K4: the fused global step (average over the replicas, sign-momentum update,
@@ -516,7 +553,7 @@ __device__ __forceinline__ void global_elem_generic(const Problem& p, const Glob
 // to one tensor and reduces them only when the tensor changes (or at its last
 // tile), writing the segment's partial at the segment's last tile and zeros
 // at its other tiles; the per-tensor sum over tiles is then unchanged.
-template <int NW>
+template <int NW, int MODE>
 __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g) {
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     constexpr int W = NW > 0 ? NW : 1;
@@ -524,22 +561,24 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
     if (ti >= p.num_tiles) return;
     TileDesc nt = p.tiles[ti];
     bool nvec = NW > 0 && vector_ok(nt, e0);
-    float x[4], m[4], r[W][4];
+    float x[4], m[4], v[4] = {0.f, 0.f, 0.f, 0.f}, r[W][4];
     ThreadStats st;
     if (nvec) {
         load4(p.x + nt.start + e0, x);
         load4(p.m + nt.start + e0, m);
+        if (MODE == 4) load4(p.gv + nt.start + e0, v);
 #pragma unroll
         for (int i = 0; i < W; ++i) load4(p.X + i * p.d_stride + nt.start + e0, r[i]);
     }
     for (; ti < p.num_tiles; ti += gridDim.x) {
         const TileDesc td = nt;
         const bool vec = nvec;
-        float cx[4], cm[4], cr[W][4];
+        float cx[4], cm[4], cv[4], cr[W][4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             cx[j] = x[j];
             cm[j] = m[j];
+            cv[j] = v[j];
 #pragma unroll
             for (int i = 0; i < W; ++i) cr[i][j] = r[i][j];
         }
@@ -550,6 +589,7 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
             if (nvec) {
                 load4(p.x + nt.start + e0, x);
                 load4(p.m + nt.start + e0, m);
+                if (MODE == 4) load4(p.gv + nt.start + e0, v);
 #pragma unroll
                 for (int i = 0; i < W; ++i) load4(p.X + i * p.d_stride + nt.start + e0, r[i]);
             }
@@ -558,7 +598,7 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
         if (vec) {
             const uint64_t gi = td.start + e0;  // a multiple of 4: the four words of one Philox block
             float ru[4] = {0.f, 0.f, 0.f, 0.f};
-            if (g.sign_mode != 0) {
+            if (MODE == 0 && g.sign_mode != 0) {
                 const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
                 ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
             }
@@ -567,15 +607,16 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
                 float dif[W];
 #pragma unroll
                 for (int i = 0; i < W; ++i) dif[i] = __fsub_rn(cx[j], cr[i][j]);
-                global_elem<W>(cx[j], cm[j], dif, W, g, lam, ru[j], st);
+                global_elem<W, MODE>(cx[j], cm[j], cv[j], dif, W, g, lam, ru[j], st);
             }
             store4(p.x + gi, cx);
             store4(p.m + gi, cm);
+            if (MODE == 4) store4(p.gv + gi, cv);
 #pragma unroll
             for (int i = 0; i < W; ++i) store4(p.X + i * p.d_stride + gi, cx);
         } else {
             const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
-            for (uint32_t e = e0; e < e1; ++e) global_elem_generic(p, g, lam, td.start + e, st);
+            for (uint32_t e = e0; e < e1; ++e) global_elem_generic<MODE>(p, g, lam, td.start + e, st);
         }
         if (next >= p.num_tiles || nt.tensor != td.tensor) {  // uniform across the CTA
             reduce_stats(st, p.partials + ti);
@@ -629,17 +670,28 @@ int grid_for(K kernel, int sms) {
 
 using GlobalKernel = void (*)(Problem, GlobalScalars);
 
-GlobalKernel global_kernel_for(uint32_t n) {
+template <int MODE>
+GlobalKernel global_kernel_mode(uint32_t n) {
     switch (n) {
-        case 1: return k_global<1>;
-        case 2: return k_global<2>;
-        case 3: return k_global<3>;
-        case 4: return k_global<4>;
-        case 5: return k_global<5>;
-        case 6: return k_global<6>;
-        case 7: return k_global<7>;
-        case 8: return k_global<8>;
-        default: return k_global<0>;
+        case 1: return k_global<1, MODE>;
+        case 2: return k_global<2, MODE>;
+        case 3: return k_global<3, MODE>;
+        case 4: return k_global<4, MODE>;
+        case 5: return k_global<5, MODE>;
+        case 6: return k_global<6, MODE>;
+        case 7: return k_global<7, MODE>;
+        case 8: return k_global<8, MODE>;
+        default: return k_global<0, MODE>;
+    }
+}
+
+GlobalKernel global_kernel_for(uint32_t n, int mode) {
+    switch (mode) {
+        case 1: return global_kernel_mode<1>(n);
+        case 2: return global_kernel_mode<2>(n);
+        case 3: return global_kernel_mode<3>(n);
+        case 4: return global_kernel_mode<4>(n);
+        default: return global_kernel_mode<0>(n);
     }
 }
 
@@ -657,7 +709,7 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms) : grid_for(k_grad_fill<false>, sms);
     out->grid_adamw = p.grad_bf16 ? grid_for(k_local_adamw<true>, sms) : grid_for(k_local_adamw<false>, sms);
     out->grid_sgdm = p.grad_bf16 ? grid_for(k_local_sgdm<true>, sms) : grid_for(k_local_sgdm<false>, sms);
-    out->grid_global = grid_for(global_kernel_for(p.n), sms);
+    out->grid_global = grid_for(global_kernel_for(p.n, p.global_mode), sms);
     return cudaGetLastError();
 }
 
@@ -700,7 +752,7 @@ cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const Sgd
 cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s) {
     const int grid = clamp_grid(ls.grid_global, p.num_tiles);
     if (grid == 0) return cudaSuccess;
-    global_kernel_for(p.n)<<<grid, kThreads, 0, s>>>(p, g);
+    global_kernel_for(p.n, p.global_mode)<<<grid, kThreads, 0, s>>>(p, g);
     return cudaGetLastError();
 }
 

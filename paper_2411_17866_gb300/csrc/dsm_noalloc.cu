@@ -144,6 +144,8 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     if (!(hp->g_eta >= 0.f && hp->g_eta < 3.0e38f) || !(hp->g_wd >= 0.f && hp->g_wd < 3.0e38f))
         return na_fail(DSM_EINVAL, "global eta and lambda must be finite and >= 0");
     if (hp->sign_mode < DSM_SIGN || hp->sign_mode > DSM_RSIGN_PM) return na_fail(DSM_EINVAL, "sign mode unknown");
+    if (hp->global_mode != DSM_GLOBAL_SIGN_MOMENTUM)
+        return na_fail(DSM_EINVAL, "only the sign-momentum global step (DSM_GLOBAL_SIGN_MOMENTUM) is available here");
     if (hp->sign_mode != DSM_SIGN && !(hp->rsign_B > 0.f && hp->rsign_B < 3.0e38f))
         return na_fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
     uint64_t d = 0, tiles = 0;
@@ -213,9 +215,10 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     p.partials = reinterpret_cast<StatPartial*>(scratch + kOffPartials);
     p.stats = reinterpret_cast<TensorStats*>(scratch + kOffStats);
 
+    p.global_mode = DSM_GLOBAL_SIGN_MOMENTUM;
     LaunchShape ls;
     if ((err = query_launch_shape(p, &ls)) != cudaSuccess) return na_cuda(err, "occupancy query");
-    GlobalScalars g;
+    GlobalScalars g{};
     g.b1 = hp->g_b1;
     g.b2 = hp->g_b2;
     g.c1 = float((1.0 - double(hp->g_b1)) / double(gamma));

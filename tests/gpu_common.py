@@ -52,6 +52,8 @@ def compare_state(run, ora, elems=None, grads=True):
         assert_bitexact(rd(dsm.BUF_OPT_M, i), ora.opt_m[i], f"opt_m {i}")
         if ora.opt_v is not None:
             assert_bitexact(rd(dsm.BUF_OPT_V, i), ora.opt_v[i], f"opt_v {i}")
+    if getattr(ora, "gv", None) is not None:
+        assert_bitexact(rd(dsm.BUF_GLOBAL_V), ora.gv, "global v")
 
 
 def compare_stats(got, want, n=64):

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(lib):
 
 def test_struct_sizes_match_header_layout():
     assert ctypes.sizeof(dsm.dsm_tensor) == 24
-    assert ctypes.sizeof(dsm.dsm_hparams) == 72
+    assert ctypes.sizeof(dsm.dsm_hparams) == 80
     assert ctypes.sizeof(dsm.dsm_tensor_stats) == 48
 
 
@@ -76,6 +76,10 @@ def test_state_bytes_covers_the_state(lib):
     (dict(hp=W.HParams(sign_mode=W.RSIGN_ZERO, rsign_B=0.0)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(grad_dtype=2)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(base=7)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(global_mode=5)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(global_mode=W.GLOBAL_SLOWMO, sign_mode=W.RSIGN_ZERO)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(global_mode=W.GLOBAL_ADAMW, g_b1=1.0)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(global_mode=W.GLOBAL_ADAMW, g_eps=0.0)), dsm.DSM_EINVAL),
     (dict(hp=W.SGDM_HP.__class__(**{**W.SGDM_HP.__dict__, "mu": 1.0})), dsm.DSM_EINVAL),
     (dict(tensors=()), dsm.DSM_EINVAL),
     (dict(tensors=(W.Tensor("z", 0, 0, 1.0),)), dsm.DSM_EINVAL),

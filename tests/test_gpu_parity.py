@@ -80,6 +80,34 @@ def test_rounds_bitexact(layout_name, name, hp, n, tau):
     run.close()
 
 
+VARIANTS = [
+    ("slowmo-adamw-n4", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO, g_b1=0.5, g_eta=0.8), 4, 2),
+    ("signed-slowmo-sgdm-n3", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_SIGNED_SLOWMO,
+                                                  g_b1=0.5, g_b2=0.5), 3, 2),
+    ("lookahead-adamw-n1", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_LOOKAHEAD, g_b1=0.2, g_b2=0.2,
+                                               g_wd=0.0, g_eta=1.0), 1, 3),
+    ("lookahead-sgdm-n8", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_LOOKAHEAD), 8, 1),
+    ("global-adamw-bf16-n4", dataclasses.replace(ADAMW, grad_dtype=W.BF16, global_mode=W.GLOBAL_ADAMW), 4, 2),
+    ("global-adamw-n9-generic", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_ADAMW), 9, 1),
+    ("slowmo-n16-generic", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_SLOWMO), 16, 1),
+]
+
+
+@pytest.mark.parametrize("layout_name", ["ragged", "mini"])
+@pytest.mark.parametrize("name,hp,n,tau", VARIANTS, ids=[c[0] for c in VARIANTS])
+def test_global_variants_bitexact(layout_name, name, hp, n, tau):
+    """The ablations' global steps (SlowMo, signed SlowMo, Lookahead, global AdamW), three rounds."""
+    tensors = RAGGED if layout_name == "ragged" else MINI
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    for _ in range(3):
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+        compare_state(run, ora)
+        compare_stats(stats, ora.last_stats, n)
+    run.close()
+
+
 def test_caller_gradients_host_and_device():
     """dsm_load_grads: gradients written by the caller (pinned host and device)."""
     tensors, n, tau = MINI, 3, 2
