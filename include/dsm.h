@@ -248,6 +248,18 @@ int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64
 int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src, uint64_t offset,
                      uint64_t count, int src_is_device, dsm_stream_t stream);
 
+/* The paper's learning-rate schedule (Sec. 5, implementations): linear
+ * warm-up to `peak` over `warmup_steps` local steps (step s < warmup_steps
+ * gives peak*(s+1)/warmup_steps), then a cosine decay to final_ratio*peak at
+ * `total_steps` (final_ratio*peak + (peak - final_ratio*peak)*(1 + cos(pi*r))/2
+ * with r = (s - warmup_steps)/(total_steps - warmup_steps)), constant after.
+ * Algorithm 1 keeps gamma_t fixed within a round: pass step = t*tau and give
+ * the result to dsm_set_gamma.  Computed in double, returned as fp32 in
+ * *gamma.  DSM_EINVAL if peak <= 0, final_ratio outside [0, 1],
+ * warmup_steps > total_steps or total_steps = 0. */
+int dsm_cosine_gamma(float peak, float final_ratio, uint64_t warmup_steps, uint64_t total_steps, uint64_t step,
+                     float* gamma);
+
 /* Set the round counter t (checkpoint restore); only between rounds. */
 int dsm_set_round(dsm_handle* h, uint64_t round);
 

@@ -219,6 +219,19 @@ def beta_power(beta: float, j: int) -> float:
     return p
 
 
+def cosine_gamma(peak: float, final_ratio: float, warmup: int, total: int, step: int) -> float:
+    """Learning rate at local step ``step`` of the paper's schedule (Sec. 5, implementations):
+    linear warm-up over ``warmup`` steps to ``peak``, then a cosine decay to final_ratio * peak at
+    ``total`` steps, constant after.  Algorithm 1's gamma_t of round t is the value at step t*tau."""
+    final = final_ratio * peak
+    if step < warmup:
+        return peak * (step + 1) / warmup
+    if step >= total:
+        return final
+    ratio = (step - warmup) / (total - warmup)
+    return final + 0.5 * (1.0 + np.cos(np.pi * ratio)) * (peak - final)
+
+
 # ---------------------------------------------------------------------------
 # Base optimizers (Appendix A) as local steps, Eq. (local-steps)
 # ---------------------------------------------------------------------------

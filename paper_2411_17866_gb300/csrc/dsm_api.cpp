@@ -524,6 +524,27 @@ int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src,
     return DSM_OK;
 }
 
+int dsm_cosine_gamma(float peak, float final_ratio, uint64_t warmup_steps, uint64_t total_steps, uint64_t step,
+                     float* gamma) {
+    if (!gamma) return fail(DSM_EINVAL, "gamma must not be NULL");
+    if (!(finite(peak) && peak > 0.f)) return fail(DSM_EINVAL, "peak must be finite and > 0");
+    if (!(final_ratio >= 0.f && final_ratio <= 1.f)) return fail(DSM_EINVAL, "final_ratio must lie in [0, 1]");
+    if (total_steps == 0 || warmup_steps > total_steps)
+        return fail(DSM_EINVAL, "need 0 < total_steps and warmup_steps <= total_steps");
+    const double P = peak, F = double(final_ratio) * double(peak);
+    double g;
+    if (step < warmup_steps) {
+        g = P * double(step + 1) / double(warmup_steps);
+    } else if (step >= total_steps) {
+        g = F;
+    } else {
+        const double r = double(step - warmup_steps) / double(total_steps - warmup_steps);
+        g = F + 0.5 * (1.0 + std::cos(M_PI * r)) * (P - F);
+    }
+    *gamma = float(g);
+    return DSM_OK;
+}
+
 int dsm_set_round(dsm_handle* h, uint64_t round) {
     if (!h) return fail(DSM_EINVAL, "handle is NULL");
     if (h->k != 0) return fail(DSM_ESTATE, "the round counter can change only between rounds");

@@ -79,6 +79,7 @@ _PROTOS = {
     "dsm_read_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
     "dsm_write_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
     "dsm_set_round": (c_int, [c_void_p, c_uint64]),
+    "dsm_cosine_gamma": (c_int, [c_float, c_float, c_uint64, c_uint64, c_uint64, POINTER(c_float)]),
     "dsm_get_info": (c_int, [c_void_p, POINTER(dsm_info)]),
     "dsm_destroy": (c_int, [c_void_p]),
     "dsm_last_error": (c_char_p, []),
@@ -226,6 +227,13 @@ def dsm_write_params(h, which: int, worker: int, src_ptr: int, offset: int, coun
 
 def dsm_set_round(h, round_: int) -> None:
     _check(load_library().dsm_set_round(h, round_), "dsm_set_round")
+
+
+def dsm_cosine_gamma(peak: float, final_ratio: float, warmup_steps: int, total_steps: int, step: int) -> float:
+    out = c_float()
+    _check(load_library().dsm_cosine_gamma(peak, final_ratio, warmup_steps, total_steps, step, byref(out)),
+           "dsm_cosine_gamma")
+    return out.value
 
 
 def dsm_get_info(h) -> dsm_info:

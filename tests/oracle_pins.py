@@ -533,9 +533,25 @@ def pin_global_adamw_vs_torch(o):
         assert np.allclose(run.x, p.detach().numpy(), rtol=1e-10, atol=1e-12)
 
 
+def pin_cosine_schedule(o):
+    """Closed-form points of warm-up + cosine decay: P/W at step 0, P at the end of the warm-up,
+    (P + F)/2 halfway through the decay, F at and after the last step; monotone decay."""
+    P, r, W_, S = 6e-4, 0.05, 2000, 100000
+    F = r * P
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, 0), P / W_, rtol=1e-15)
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, W_ - 1), P, rtol=1e-15)
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, W_), P, rtol=1e-15)
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, (W_ + S) // 2), (P + F) / 2, rtol=1e-12)
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, S), F, rtol=1e-15)
+    assert np.isclose(o.cosine_gamma(P, r, W_, S, 10 * S), F, rtol=1e-15)
+    vals = [o.cosine_gamma(P, r, W_, S, s) for s in range(W_, S + 1, 997)]
+    assert all(a >= b for a, b in zip(vals, vals[1:]))
+
+
 PINS = [pin_worked_example, pin_splitmix64, pin_philox, pin_philox_uniform_mapping, pin_bf16,
         pin_uniform24, pin_hash_fields, pin_synthetic_grad, pin_adamw_vs_torch, pin_adamw_constant_grad,
         pin_adamw_first_step_fp32, pin_sgdm_vs_torch, pin_sgd_plain_exact, pin_sgdm_constant_grad,
         pin_lion, pin_signsgd_momentum, pin_identical_workers, pin_tau1_pseudo_gradient,
         pin_sign_range, pin_lemma1, pin_stats, pin_subset_mode, pin_fp32_vs_fp64,
-        pin_slowmo_heavy_ball, pin_lookahead_slow_weights, pin_signed_slowmo_signsgd, pin_global_adamw_vs_torch]
+        pin_slowmo_heavy_ball, pin_lookahead_slow_weights, pin_signed_slowmo_signsgd, pin_global_adamw_vs_torch,
+        pin_cosine_schedule]

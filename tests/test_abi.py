@@ -129,3 +129,17 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(dsm, "_lib", None)
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         dsm.load_library(str(tmp_path / "missing.so"))
+
+
+def test_cosine_schedule_matches_the_oracle(lib):
+    """dsm_cosine_gamma against the oracle's schedule (itself pinned by closed-form points)."""
+    import numpy as np
+    from oracle import dsm_oracle as O
+    P, r, W_, S = 6e-4, 0.05, 2000, 100000
+    for step in list(range(0, 2100, 7)) + list(range(2000, 100001, 991)) + [100000, 100001, 10 ** 9]:
+        want = np.float32(O.cosine_gamma(P, r, W_, S, step))
+        got = np.float32(dsm.dsm_cosine_gamma(P, r, W_, S, step))
+        assert abs(int(got.view(np.int32)) - int(want.view(np.int32))) <= 1, (step, got, want)
+    for bad in [(0.0, r, W_, S, 0), (P, 1.5, W_, S, 0), (P, r, S + 1, S, 0), (P, r, 0, 0, 0)]:
+        with pytest.raises(dsm.DsmError):
+            dsm.dsm_cosine_gamma(*bad)
