@@ -3,6 +3,9 @@
 A step is one global round of Algorithm 1 on the synthetic workload: tau
 times (synthetic gradient fill for all n workers + one local base-optimizer
 step on all n replicas), then the fused global step and its statistics.
+By default the round is fused (the last local step runs inside the global
+step and the replica reset is deferred to the next round's first local
+step); --no-fused runs every step separately.  Both give identical results.
 All inputs are resident in HBM when the timed region starts.
 
 Metric: params/s per global round = d x rounds / device time (whole job).
@@ -58,6 +61,8 @@ def parse():
     ap.add_argument("--max-params", type=int, default=None)
     # the global step: Algorithm 1 (default) or a variant of the ablations
     ap.add_argument("--global-mode", default=None, choices=sorted(GLOBAL_MODES))
+    # fused round (default): the last local step inside the global step, lazy replica reset
+    ap.add_argument("--no-fused", dest="fused", action="store_false")
     return ap.parse_args()
 
 
@@ -82,6 +87,11 @@ def select_workload(args):
         changes["hp"] = dataclasses.replace(wl.hp, global_mode=mode,
                                             sign_mode=wl.hp.sign_mode if mode == W.GLOBAL_SIGN_MOMENTUM else W.SIGN)
         notes.append(f"global step {args.global_mode}")
+    if args.fused:   # an execution option: the results are bit-identical to the unfused round
+        hp = changes.get("hp", wl.hp)
+        changes["hp"] = dataclasses.replace(hp, flags=hp.flags | W.FLAG_FUSED_ROUND)
+    else:
+        notes.append("unfused round")
     if args.max_params:
         keep, total = [], 0
         for t in wl.tensors:
@@ -137,6 +147,19 @@ def bytes_per_elem_local(wl) -> int:
 def bytes_per_param_global(wl) -> int:
     # read x, m (and the global AdamW second moment) and n replicas; write them all
     return 8 * (wl.n + 2 + (1 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0))
+
+
+def fused_round_active(wl) -> bool:
+    """The library fuses the round for the sign-momentum global step with n <= 8."""
+    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.hp.global_mode == W.GLOBAL_SIGN_MOMENTUM and wl.n <= 8
+
+
+def bytes_per_param_fused_last(wl) -> int:
+    """Fused last local step + global step: per worker read x_i, the optimizer state and g and write the
+    state back (x_i is not written); read and write x and m; no replica reset."""
+    g = 2 if wl.hp.grad_dtype == W.BF16 else 4
+    states = 2 if wl.hp.base == W.BASE_ADAMW else 1
+    return wl.n * (4 + 8 * states + g) + 16
 
 
 def measured_peaks():
@@ -268,6 +291,7 @@ def workload_config(wl, gpus):
             "grad_dtype": "bf16" if wl.hp.grad_dtype == W.BF16 else "f32",
             "sign": ["sign", "rand-sign-2", "rand-sign-1"][wl.hp.sign_mode],
             "global_step": {v: k for k, v in GLOBAL_MODES.items()}[wl.hp.global_mode],
+            "fused_round": bool(wl.hp.flags & W.FLAG_FUSED_ROUND),
             "parallelism": f"param-shard x{gpus}" if gpus > 1 else "single GPU",
             "l2": "inputs larger than L2 (129 MB): each local-step launch streams "
                   f"{wl.n * wl.d * bytes_per_elem_local(wl) / 1e9:.1f} GB"}
@@ -293,16 +317,22 @@ def main():
     stream = torch.cuda.current_stream(dev)
     tau = wl.tau
 
+    fused = fused_round_active(wl)
+    local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
+    local_bytes_from_x = wl.n * wl.d * (bytes_per_elem_local(wl) - 4) + wl.d * 4
+
     def round_(t, local_events=None, global_events=None):
         for k in range(tau):
             run.fill_synthetic_grads(t * tau + k, stream)
-            if local_events is not None:
+            if local_events is not None and not (fused and k == tau - 1):
                 a = torch.cuda.Event(enable_timing=True)
                 b = torch.cuda.Event(enable_timing=True)
                 a.record(stream)
                 run.local_step(stream)
                 b.record(stream)
-                local_events.append((a, b))
+                # fused round: the first local step starts every worker from x (read once per tile)
+                nbytes = local_bytes_from_x if (fused and k == 0 and t > 0) else local_bytes
+                local_events.append((a, b, nbytes))
             else:
                 run.local_step(stream)
         if global_events is not None:
@@ -340,7 +370,8 @@ def main():
         dist.barrier()
     clocks = sampler.stop() if sampler else None
     elapsed = max_over_ranks(start.elapsed_time(end) / 1e3, world)
-    local_ms = [a.elapsed_time(b) for a, b in local_ev]
+    local_ms = [a.elapsed_time(b) for a, b, _ in local_ev]
+    local_launch_bytes = [nb for _, _, nb in local_ev]
     global_ms = [a.elapsed_time(b) for a, b in global_ev]
 
     # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device
@@ -377,12 +408,12 @@ def main():
         return 0
 
     peak, peak_kind = measured_peaks()
-    local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
+    # fused round: the last local step runs inside the global-step launch
+    global_bytes = wl.d * (bytes_per_param_global(wl) if not fused else bytes_per_param_fused_last(wl))
     avg_local_s = statistics.mean(local_ms) / 1e3
-    achieved = local_bytes / avg_local_s / 1e9
+    achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
     kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
     traffic = committed_traffic(f"{kname}:{args.workload}")
-    global_bytes = wl.d * bytes_per_param_global(wl)
     avg_global_s = statistics.mean(global_ms) / 1e3
     value = whole_job_value(wl.d, world, args.steps, elapsed)
     line = {
@@ -397,9 +428,11 @@ def main():
         "global_step": {"bytes_per_launch": global_bytes, "avg_ms": avg_global_s * 1e3,
                         "achieved_gbs": global_bytes / avg_global_s / 1e9,
                         "frac": global_bytes / avg_global_s / 1e9 / peak,
-                        "note": "fused global step + statistics reduction, CUDA events around both"},
+                        "note": ("last local step fused with the global step, + statistics reduction"
+                                 if fused else "fused global step + statistics reduction") +
+                                ", CUDA events around both"},
         "optimizer_only_value": wl.d * args.steps / ((sum(local_ms) + sum(global_ms)) / 1e3),
-        "gpu_launches": args.steps * (2 * tau + 2),
+        "gpu_launches": args.steps * (2 * tau + (1 if fused else 2)),
         "e2e": e2e,
         "clocks": clocks,
     }

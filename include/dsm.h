@@ -94,6 +94,19 @@ extern "C" {
 #define DSM_GLOBAL_LOOKAHEAD     3
 #define DSM_GLOBAL_ADAMW         4
 
+/* Fused round.  Same results, fewer bytes: the round's last local step
+ * runs inside dsm_global_step (dsm_local_step for k = tau-1 only records
+ * it), so its new replicas never go to memory, and the reset of the replicas
+ * is lazy: the next round's first local step starts every worker from x
+ * instead of reading n copies of it.  Applies to the sign-momentum global
+ * step with n <= 8; other settings run unfused.  Reading a replica while
+ * the reset is pending returns x; reading or writing worker state, or
+ * writing gradients through dsm_fill_synthetic_grads/dsm_load_grads, while
+ * the last local step is pending first runs that step unfused.  Gradients
+ * written through dsm_grad_ptr must not change between the last
+ * dsm_local_step and dsm_global_step. */
+#define DSM_FLAG_FUSED_ROUND 1u
+
 /* Buffers for dsm_read_params / dsm_write_params. */
 #define DSM_BUF_X        0  /* global model x_{t,0} (fp32, d) */
 #define DSM_BUF_M        1  /* global momentum m_t (fp32, d) */
@@ -135,7 +148,7 @@ typedef struct {
     int32_t sign_mode;   /* DSM_SIGN | DSM_RSIGN_ZERO | DSM_RSIGN_PM */
     float rsign_B;       /* bound B of Eqs. (rand-sign-1/2); > 0 when randomized */
     int32_t grad_dtype;  /* DSM_F32 | DSM_BF16 */
-    uint32_t reserved;   /* must be 0 */
+    uint32_t flags;      /* DSM_FLAG_* bits; others must be 0 */
     uint64_t seed;       /* seed of the synthetic generators and of the Philox key */
     int32_t global_mode; /* DSM_GLOBAL_* */
     float g_eps;         /* epsilon of the global AdamW step, > 0 when global_mode is DSM_GLOBAL_ADAMW */

@@ -101,7 +101,7 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
         return fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
     if (hp->grad_dtype != DSM_F32 && hp->grad_dtype != DSM_BF16)
         return fail(DSM_EINVAL, "gradient dtype %d unknown", hp->grad_dtype);
-    if (hp->reserved != 0) return fail(DSM_EINVAL, "hparams.reserved must be 0");
+    if (hp->flags & ~DSM_FLAG_FUSED_ROUND) return fail(DSM_EINVAL, "unknown bits in hparams.flags");
 
     uint64_t d = 0, tiles = 0;
     for (uint32_t i = 0; i < layout->count; ++i) {
@@ -180,6 +180,12 @@ struct dsm_handle {
     double b2_pow = 1.0;
     double gb1_pow = 1.0;  // global AdamW: beta1^t and beta2^t after t global steps
     double gb2_pow = 1.0;
+    // fused round (DSM_FLAG_FUSED_ROUND)
+    bool fused = false;           // flag set and a fused kernel exists for this problem
+    bool replicas_stale = false;  // the replicas' reset to x is pending
+    bool last_pending = false;    // the round's last local step waits for the global step
+    AdamScalars pending_a{};
+    SgdmScalars pending_sa{};
     uint64_t j = 0;        // local steps done since the start (AdamW step count)
 };
 
@@ -225,6 +231,55 @@ int copy_kind(const void* host_or_dev, int is_device, bool to_device, cudaMemcpy
     (void)host_or_dev;
     if (to_device) *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     else *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+    return DSM_OK;
+}
+
+// Scalars of the next local step (count j + 1); advances the beta powers.
+void next_local_scalars(dsm_handle* h, AdamScalars* a, SgdmScalars* sa) {
+    *a = AdamScalars{};
+    *sa = SgdmScalars{};
+    if (h->hp.base == DSM_BASE_ADAMW) {
+        const double nb1 = h->b1_pow * double(h->hp.b1);
+        const double nb2 = h->b2_pow * double(h->hp.b2);
+        a->b1 = h->hp.b1;
+        a->omb1 = float(1.0 - double(h->hp.b1));
+        a->b2 = h->hp.b2;
+        a->omb2 = float(1.0 - double(h->hp.b2));
+        a->bc1 = float(1.0 - nb1);
+        a->bc2 = float(1.0 - nb2);
+        a->lr = h->gamma;
+        a->eps = h->hp.eps;
+        h->b1_pow = nb1;
+        h->b2_pow = nb2;
+    } else {
+        sa->mu = h->hp.mu;
+        sa->lr = h->gamma;
+    }
+}
+
+cudaError_t launch_local(dsm_handle* h, const AdamScalars& a, const SgdmScalars& sa, cudaStream_t s) {
+    const bool from_x = h->replicas_stale;
+    cudaError_t err = h->hp.base == DSM_BASE_ADAMW ? launch_local_adamw(h->prob, h->shape, a, from_x, s)
+                                                   : launch_local_sgdm(h->prob, h->shape, sa, from_x, s);
+    if (err == cudaSuccess) h->replicas_stale = false;
+    return err;
+}
+
+// Runs a deferred last local step unfused (before its inputs or outputs are touched).
+int materialize_pending(dsm_handle* h, cudaStream_t s) {
+    if (!h->last_pending) return DSM_OK;
+    cudaError_t err = launch_local(h, h->pending_a, h->pending_sa, s);
+    if (err != cudaSuccess) return cuda_fail(err, "launch the deferred local step");
+    h->last_pending = false;
+    return DSM_OK;
+}
+
+// Writes x into every replica (the reset the fused round left pending).
+int materialize_replicas(dsm_handle* h, cudaStream_t s) {
+    if (!h->replicas_stale) return DSM_OK;
+    cudaError_t err = launch_init(h->prob, h->shape, 0, 0, s);
+    if (err != cudaSuccess) return cuda_fail(err, "reset the replicas");
+    h->replicas_stale = false;
     return DSM_OK;
 }
 
@@ -330,6 +385,7 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
         return cuda_fail(e, what);
     };
     if ((err = query_launch_shape(p, &h->shape)) != cudaSuccess) return bail(err, "occupancy query");
+    h->fused = (hp->flags & DSM_FLAG_FUSED_ROUND) && fused_round_available(p);
     // The tables are copied from the handle's own vectors, which outlive the copies.
     if ((err = cudaMemcpyAsync(A + al.off_tensors, h->tensors.data(), h->tensors.size() * sizeof(TensorDesc),
                                cudaMemcpyHostToDevice, s)) != cudaSuccess)
@@ -367,6 +423,8 @@ int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream) 
     for (uint32_t i = 0; i < kMaxWorkers; ++i) k.worker[i] = i < h->n ? draw_key(h->hp.seed, 1, i) : 0;
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    int rc = materialize_pending(h, S(stream));
+    if (rc != DSM_OK) return rc;
     cudaError_t err = launch_grad_fill(h->prob, h->shape, k, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "launch grad fill");
     return DSM_OK;
@@ -383,6 +441,8 @@ int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream
     if (!h || !src) return fail(DSM_EINVAL, "NULL argument");
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    int rc = materialize_pending(h, S(stream));
+    if (rc != DSM_OK) return rc;
     const size_t es = h->al.grad_esize;
     const cudaMemcpyKind kind = src_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     cudaError_t err;
@@ -402,30 +462,17 @@ int dsm_local_step(dsm_handle* h, dsm_stream_t stream) {
                     (unsigned long long)h->t);
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
-    cudaError_t err;
-    if (h->hp.base == DSM_BASE_ADAMW) {
-        // step count j = t*tau + k + 1; beta^j by successive float64 products
-        const double nb1 = h->b1_pow * double(h->hp.b1);
-        const double nb2 = h->b2_pow * double(h->hp.b2);
-        AdamScalars a;
-        a.b1 = h->hp.b1;
-        a.omb1 = float(1.0 - double(h->hp.b1));
-        a.b2 = h->hp.b2;
-        a.omb2 = float(1.0 - double(h->hp.b2));
-        a.bc1 = float(1.0 - nb1);
-        a.bc2 = float(1.0 - nb2);
-        a.lr = h->gamma;
-        a.eps = h->hp.eps;
-        err = launch_local_adamw(h->prob, h->shape, a, S(stream));
-        if (err != cudaSuccess) return cuda_fail(err, "launch AdamW local step");
-        h->b1_pow = nb1;
-        h->b2_pow = nb2;
+    // step count j = t*tau + k + 1; beta^j by successive float64 products
+    AdamScalars a;
+    SgdmScalars sa;
+    next_local_scalars(h, &a, &sa);
+    if (h->fused && h->k + 1 == h->tau) {  // the last step runs inside dsm_global_step
+        h->pending_a = a;
+        h->pending_sa = sa;
+        h->last_pending = true;
     } else {
-        SgdmScalars a;
-        a.mu = h->hp.mu;
-        a.lr = h->gamma;
-        err = launch_local_sgdm(h->prob, h->shape, a, S(stream));
-        if (err != cudaSuccess) return cuda_fail(err, "launch SGD-momentum local step");
+        cudaError_t err = launch_local(h, a, sa, S(stream));
+        if (err != cudaSuccess) return cuda_fail(err, "launch local step");
     }
     h->j += 1;
     h->k += 1;
@@ -462,8 +509,18 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     g.philox_k0 = static_cast<uint32_t>(h->hp.seed & 0xFFFFFFFFull);
     g.philox_k1 = static_cast<uint32_t>(h->t & 0xFFFFFFFFull);
     cudaStream_t s = S(stream);
-    cudaError_t err = launch_global(h->prob, h->shape, g, s);
-    if (err != cudaSuccess) return cuda_fail(err, "launch global step");
+    cudaError_t err;
+    if (h->last_pending) {  // fused round: last local step + global step, reset left pending
+        err = launch_fused_last_global(h->prob, h->shape, h->pending_a, h->pending_sa, g, h->replicas_stale, s);
+        if (err != cudaSuccess) return cuda_fail(err, "launch fused last local step and global step");
+        h->last_pending = false;
+        h->replicas_stale = true;
+    } else {
+        int rc = materialize_replicas(h, s);
+        if (rc != DSM_OK) return rc;
+        err = launch_global(h->prob, h->shape, g, s);
+        if (err != cudaSuccess) return cuda_fail(err, "launch global step");
+    }
     err = launch_stats(h->prob, s);
     if (err != cudaSuccess) return cuda_fail(err, "launch statistics");
     h->t += 1;
@@ -496,6 +553,11 @@ int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64
     if (count == 0) return DSM_OK;
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    if (which >= DSM_BUF_REPLICA && which <= DSM_BUF_OPT_V) {
+        rc = materialize_pending(h, S(stream));
+        if (rc != DSM_OK) return rc;
+    }
+    if (which == DSM_BUF_REPLICA && h->replicas_stale) src = reinterpret_cast<char*>(h->prob.x + offset);
     cudaMemcpyKind kind;
     copy_kind(dst, dst_is_device, false, &kind);
     cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
@@ -515,6 +577,8 @@ int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src,
     if (count == 0) return DSM_OK;
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    if ((rc = materialize_pending(h, S(stream))) != DSM_OK) return rc;
+    if ((rc = materialize_replicas(h, S(stream))) != DSM_OK) return rc;
     cudaMemcpyKind kind;
     copy_kind(src, src_is_device, true, &kind);
     cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));

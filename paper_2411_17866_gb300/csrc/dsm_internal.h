@@ -115,6 +115,7 @@ struct GradKeys {
 struct LaunchShape {
     int sms = 0;
     int grid_grad = 0, grid_adamw = 0, grid_sgdm = 0, grid_global = 0, grid_init = 0;
+    int grid_fused = 0, grid_adamw_from_x = 0, grid_sgdm_from_x = 0;
 };
 
 // Launchers (dsm_kernels.cu).  Each returns the cudaError_t of its launch.
@@ -122,8 +123,15 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out);
 cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t seed_key_init, int from_hash,
                         cudaStream_t s);
 cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s);
-cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, cudaStream_t s);
-cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, cudaStream_t s);
+// from_x: every worker starts from the global x (the replicas' reset is pending).
+cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, bool from_x,
+                               cudaStream_t s);
+cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, bool from_x,
+                              cudaStream_t s);
+// The fused round's last local step + sign-momentum global step (n <= 8).
+bool fused_round_available(const Problem& p);
+cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
+                                     const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s);
 cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);
 cudaError_t launch_stats(const Problem& p, cudaStream_t s);
 

@@ -396,19 +396,32 @@ __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
     }
 }
 
-// Where a local-step work item (worker w, tile) lives.
+// Where a local-step work item (worker w, tile) lives.  Items are worker-major
+// (all tiles of worker 0, then worker 1, ...), or tile-major when the step
+// starts every worker from the global x (the workers of one tile then run
+// together and read that tile of x once from HBM).
 struct LocalItem {
     uint64_t base;   // w * d_stride + tile start
+    uint64_t start;  // tile start (offset in x)
     uint32_t len;
     float lam;
     bool vec;
 };
 
+template <bool kTileMajor>
 __device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t item, uint32_t e0, bool local_lam) {
-    const uint32_t w = item / p.num_tiles;
-    const TileDesc td = p.tiles[item - w * p.num_tiles];
+    uint32_t w, ti;
+    if (kTileMajor) {
+        ti = item / p.n;
+        w = item - ti * p.n;
+    } else {
+        w = item / p.num_tiles;
+        ti = item - w * p.num_tiles;
+    }
+    const TileDesc td = p.tiles[ti];
     LocalItem it;
     it.base = w * p.d_stride + td.start;
+    it.start = td.start;
     it.len = td.len;
     it.lam = local_lam ? p.tensors[td.tensor].lam_local : 0.f;
     it.vec = vector_ok(td, e0);
@@ -416,17 +429,18 @@ __device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t item,
 }
 
 // K2: one AdamW local step on every worker (work item = (worker, tile)),
-// double-buffered in registers.
-template <bool kBf16>
+// double-buffered in registers.  kFromGlobal: every worker starts from the
+// global x (the replicas' reset is still pending).
+template <bool kBf16, bool kFromGlobal>
 __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars a) {
     const uint32_t items = p.num_tiles * p.n;
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
-    LocalItem nx = local_item(p, item, e0, true);
+    LocalItem nx = local_item<kFromGlobal>(p, item, e0, true);
     float x[4], m[4], v[4], g[4];
     if (nx.vec) {
-        load4(p.X + nx.base + e0, x);
+        load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
         load4(p.opt_m + nx.base + e0, m);
         load4(p.opt_v + nx.base + e0, v);
         load4_grad<kBf16>(p.grad, nx.base + e0, g);
@@ -438,9 +452,9 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
         for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cm[j] = m[j]; cv[j] = v[j]; cg[j] = g[j]; }
         const uint32_t next = item + gridDim.x;
         if (next < items) {  // issue the next item's loads before computing this one
-            nx = local_item(p, next, e0, true);
+            nx = local_item<kFromGlobal>(p, next, e0, true);
             if (nx.vec) {
-                load4(p.X + nx.base + e0, x);
+                load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
                 load4(p.opt_m + nx.base + e0, m);
                 load4(p.opt_v + nx.base + e0, v);
                 load4_grad<kBf16>(p.grad, nx.base + e0, g);
@@ -456,7 +470,7 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
             const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
                 const uint64_t i = cur.base + e;
-                float xs = p.X[i], ms = p.opt_m[i], vs = p.opt_v[i];
+                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i], ms = p.opt_m[i], vs = p.opt_v[i];
                 adamw_elem(xs, ms, vs, load_grad1(p.grad, kBf16, i), a, cur.lam);
                 p.X[i] = xs; p.opt_m[i] = ms; p.opt_v[i] = vs;
             }
@@ -465,16 +479,16 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
 }
 
 // K3: one SGD-momentum local step on every worker, double-buffered.
-template <bool kBf16>
+template <bool kBf16, bool kFromGlobal>
 __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars a) {
     const uint32_t items = p.num_tiles * p.n;
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
-    LocalItem nx = local_item(p, item, e0, false);
+    LocalItem nx = local_item<kFromGlobal>(p, item, e0, false);
     float x[4], b[4], g[4];
     if (nx.vec) {
-        load4(p.X + nx.base + e0, x);
+        load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
         load4(p.opt_m + nx.base + e0, b);
         load4_grad<kBf16>(p.grad, nx.base + e0, g);
     }
@@ -485,9 +499,9 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
         for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cb[j] = b[j]; cg[j] = g[j]; }
         const uint32_t next = item + gridDim.x;
         if (next < items) {
-            nx = local_item(p, next, e0, false);
+            nx = local_item<kFromGlobal>(p, next, e0, false);
             if (nx.vec) {
-                load4(p.X + nx.base + e0, x);
+                load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
                 load4(p.opt_m + nx.base + e0, b);
                 load4_grad<kBf16>(p.grad, nx.base + e0, g);
             }
@@ -501,7 +515,7 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
             const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
                 const uint64_t i = cur.base + e;
-                float xs = p.X[i], bs = p.opt_m[i];
+                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i], bs = p.opt_m[i];
                 sgdm_elem(xs, bs, load_grad1(p.grad, kBf16, i), a);
                 p.X[i] = xs; p.opt_m[i] = bs;
             }
@@ -627,6 +641,173 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
     }
 }
 
+// Per-thread asynchronous global -> shared copies (cp.async): the copy holds
+// no register while in flight, and a thread waits only for its own groups.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// K6: the round's last local step fused with the sign-momentum global step.
+// One thread owns 4 elements of every worker: it runs the base optimizer's
+// last step on each worker (writing the worker's optimizer state, but not
+// its new replica, which only feeds the average), then the global step of
+// Algorithm 1 on those elements.  The replicas are not reset: the next
+// round's first local step starts every worker from x.  from_global: the
+// replicas' reset from the previous round is still pending (tau = 1).
+// A CTA walks its tiles worker by worker; each thread keeps the next
+// kFusedDepth (tile, worker) items in flight with cp.async into its own
+// shared-memory slots (x_i, m_i, v_i, g_i, and x, m with a tile's first worker).
+constexpr int kFusedDepth = 3;
+constexpr int kFusedStreams = 6;
+constexpr size_t kFusedSmem = size_t(kFusedDepth) * kFusedStreams * kThreads * sizeof(float4);
+
+template <bool kAdamW, bool kBf16, int NW>
+__global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
+                                                                GlobalScalars g, int from_global) {
+    extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+    auto slot = [&](int it, int stream) -> float4* {
+        return fsm + (size_t(it % kFusedDepth) * kFusedStreams + stream) * kThreads + threadIdx.x;
+    };
+    // Issue item `it` (tile number it / NW of this CTA, worker it % NW); always commits one group.
+    auto issue = [&](uint32_t it) {
+        const uint32_t q = it / NW, w = it - q * NW;
+        const uint64_t ti = blockIdx.x + uint64_t(q) * gridDim.x;
+        if (ti < p.num_tiles) {
+            const TileDesc t = p.tiles[ti];
+            if (vector_ok(t, e0)) {
+                const uint64_t gi = t.start + e0;
+                const uint64_t o = w * p.d_stride + gi;
+                if (!from_global) cp_async16(slot(it, 0), p.X + o);
+                cp_async16(slot(it, 1), p.opt_m + o);
+                if (kAdamW) cp_async16(slot(it, 2), p.opt_v + o);
+                if (kBf16) cp_async8(slot(it, 3), reinterpret_cast<const __nv_bfloat16*>(p.grad) + o);
+                else cp_async16(slot(it, 3), reinterpret_cast<const float*>(p.grad) + o);
+                if (w == 0) {
+                    cp_async16(slot(it, 4), p.x + gi);
+                    cp_async16(slot(it, 5), p.m + gi);
+                }
+            }
+        }
+        cp_async_commit();
+    };
+    auto take = [&](int it, int stream, float (&v)[4]) {
+        const float4 t = *slot(it, stream);
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+    };
+    uint32_t next_issue = 0;
+    for (int k = 0; k < kFusedDepth; ++k) issue(next_issue++);
+    ThreadStats st;
+    uint32_t it = 0;
+    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = p.tiles[ti];
+        const TensorDesc& T = p.tensors[td.tensor];
+        const float lam_l = kAdamW ? T.lam_local : 0.f, lam_g = T.lam_global;
+        const uint64_t gi = td.start + e0;
+        if (vector_ok(td, e0)) {
+            float x[4], m[4], dif[NW][4];
+#pragma unroll
+            for (int w = 0; w < NW; ++w, ++it) {
+                cp_async_wait<kFusedDepth - 1>();  // item `it` has landed
+                float xi[4], mi[4], vi[4], gr[4];
+                if (w == 0) {
+                    take(it, 4, x);
+                    take(it, 5, m);
+                }
+                if (from_global) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) xi[j] = x[j];
+                } else {
+                    take(it, 0, xi);
+                }
+                take(it, 1, mi);
+                if (kAdamW) take(it, 2, vi);
+                if (kBf16) {
+                    const uint2 raw = *reinterpret_cast<const uint2*>(slot(it, 3));
+                    gr[0] = __uint_as_float(raw.x << 16);
+                    gr[1] = __uint_as_float(raw.x & 0xFFFF0000u);
+                    gr[2] = __uint_as_float(raw.y << 16);
+                    gr[3] = __uint_as_float(raw.y & 0xFFFF0000u);
+                } else {
+                    take(it, 3, gr);
+                }
+                const uint64_t o = w * p.d_stride + gi;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (kAdamW) adamw_elem(xi[j], mi[j], vi[j], gr[j], a, lam_l);
+                    else sgdm_elem(xi[j], mi[j], gr[j], sa);
+                    dif[w][j] = __fsub_rn(x[j], xi[j]);
+                }
+                store4(p.opt_m + o, mi);
+                if (kAdamW) store4(p.opt_v + o, vi);
+                // refill the slot just read; the arithmetic above consumed its values, so the
+                // shared-memory reads are complete before the asynchronous copy can overwrite them
+                issue(next_issue++);
+            }
+            float ru[4] = {0.f, 0.f, 0.f, 0.f};
+            if (g.sign_mode != 0) {
+                const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float d[NW];
+#pragma unroll
+                for (int w = 0; w < NW; ++w) d[w] = dif[w][j];
+                float unused = 0.f;
+                global_elem<NW, 0>(x[j], m[j], unused, d, NW, g, lam_g, ru[j], st);
+            }
+            store4(p.x + gi, x);
+            store4(p.m + gi, m);
+        } else {
+            // this thread issued no copies for the tile; keep the group count in step
+#pragma unroll
+            for (int w = 0; w < NW; ++w, ++it) issue(next_issue++);
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t gj = td.start + e;
+                float x = p.x[gj], m = p.m[gj], d[NW];
+#pragma unroll
+                for (int w = 0; w < NW; ++w) {
+                    const uint64_t o = w * p.d_stride + gj;
+                    float xi = from_global ? x : p.X[o], mi = p.opt_m[o];
+                    if (kAdamW) {
+                        float vi = p.opt_v[o];
+                        adamw_elem(xi, mi, vi, load_grad1(p.grad, kBf16, o), a, lam_l);
+                        p.opt_v[o] = vi;
+                    } else {
+                        sgdm_elem(xi, mi, load_grad1(p.grad, kBf16, o), sa);
+                    }
+                    p.opt_m[o] = mi;
+                    d[w] = __fsub_rn(x, xi);
+                }
+                float r = 0.f;
+                if (g.sign_mode != 0) r = philox_unit(word_of(philox_block(gj >> 2, g.philox_k0, g.philox_k1), gj & 3));
+                float unused = 0.f;
+                global_elem<NW, 0>(x, m, unused, d, NW, g, lam_g, r, st);
+                p.x[gj] = x;
+                p.m[gj] = m;
+            }
+        }
+        const uint32_t next = ti + gridDim.x;
+        if (next >= p.num_tiles || p.tiles[next].tensor != td.tensor) {  // uniform across the CTA
+            reduce_stats(st, p.partials + ti);
+            st = ThreadStats();
+        } else {
+            zero_partial(p.partials + ti);
+        }
+    }
+    cp_async_wait<0>();  // the groups issued past the last tile are empty; nothing is left in flight
+}
+
 // K5: per-tensor statistics from the tile partials, in a fixed order.
 __global__ void __launch_bounds__(kThreads) k_stats(Problem p) {
     const uint32_t T = blockIdx.x;
@@ -661,9 +842,9 @@ __global__ void __launch_bounds__(kThreads) k_stats(Problem p) {
 }
 
 template <typename K>
-int grid_for(K kernel, int sms) {
+int grid_for(K kernel, int sms, size_t smem = 0) {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, 0) != cudaSuccess || per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem) != cudaSuccess || per_sm < 1)
         per_sm = 1;
     return sms * per_sm;
 }
@@ -695,7 +876,33 @@ GlobalKernel global_kernel_for(uint32_t n, int mode) {
     }
 }
 
+using FusedKernel = void (*)(Problem, AdamScalars, SgdmScalars, GlobalScalars, int);
+
+template <bool kAdamW, bool kBf16>
+FusedKernel fused_kernel_n(uint32_t n) {
+    switch (n) {
+        case 1: return k_fused_last_global<kAdamW, kBf16, 1>;
+        case 2: return k_fused_last_global<kAdamW, kBf16, 2>;
+        case 3: return k_fused_last_global<kAdamW, kBf16, 3>;
+        case 4: return k_fused_last_global<kAdamW, kBf16, 4>;
+        case 5: return k_fused_last_global<kAdamW, kBf16, 5>;
+        case 6: return k_fused_last_global<kAdamW, kBf16, 6>;
+        case 7: return k_fused_last_global<kAdamW, kBf16, 7>;
+        case 8: return k_fused_last_global<kAdamW, kBf16, 8>;
+        default: return nullptr;
+    }
+}
+
+FusedKernel fused_kernel_for(const Problem& p, bool adamw) {
+    if (adamw) return p.grad_bf16 ? fused_kernel_n<true, true>(p.n) : fused_kernel_n<true, false>(p.n);
+    return p.grad_bf16 ? fused_kernel_n<false, true>(p.n) : fused_kernel_n<false, false>(p.n);
+}
+
 }  // namespace
+
+bool fused_round_available(const Problem& p) {
+    return p.global_mode == 0 && p.n >= 1 && p.n <= kMaxUnrolledWorkers;
+}
 
 cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     int dev = 0;
@@ -707,8 +914,16 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     out->sms = sms;
     out->grid_init = grid_for(k_init, sms);
     out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms) : grid_for(k_grad_fill<false>, sms);
-    out->grid_adamw = p.grad_bf16 ? grid_for(k_local_adamw<true>, sms) : grid_for(k_local_adamw<false>, sms);
-    out->grid_sgdm = p.grad_bf16 ? grid_for(k_local_sgdm<true>, sms) : grid_for(k_local_sgdm<false>, sms);
+    out->grid_adamw = p.grad_bf16 ? grid_for(k_local_adamw<true, false>, sms) : grid_for(k_local_adamw<false, false>, sms);
+    out->grid_sgdm = p.grad_bf16 ? grid_for(k_local_sgdm<true, false>, sms) : grid_for(k_local_sgdm<false, false>, sms);
+    if (fused_round_available(p)) {
+        const FusedKernel fk = fused_kernel_for(p, p.opt_v != nullptr);
+        cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kFusedSmem));
+        if (e != cudaSuccess) return e;
+        out->grid_fused = grid_for(fk, sms, kFusedSmem);
+        out->grid_adamw_from_x = p.grad_bf16 ? grid_for(k_local_adamw<true, true>, sms) : grid_for(k_local_adamw<false, true>, sms);
+        out->grid_sgdm_from_x = p.grad_bf16 ? grid_for(k_local_sgdm<true, true>, sms) : grid_for(k_local_sgdm<false, true>, sms);
+    }
     out->grid_global = grid_for(global_kernel_for(p.n, p.global_mode), sms);
     return cudaGetLastError();
 }
@@ -733,19 +948,42 @@ cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const Grad
     return cudaGetLastError();
 }
 
-cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, cudaStream_t s) {
-    const int grid = clamp_grid(ls.grid_adamw, static_cast<uint64_t>(p.num_tiles) * p.n);
+cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, bool from_x,
+                               cudaStream_t s) {
+    const uint64_t items = static_cast<uint64_t>(p.num_tiles) * p.n;
+    const int grid = clamp_grid(from_x ? ls.grid_adamw_from_x : ls.grid_adamw, items);
     if (grid == 0) return cudaSuccess;
-    if (p.grad_bf16) k_local_adamw<true><<<grid, kThreads, 0, s>>>(p, a);
-    else k_local_adamw<false><<<grid, kThreads, 0, s>>>(p, a);
+    if (from_x) {
+        if (p.grad_bf16) k_local_adamw<true, true><<<grid, kThreads, 0, s>>>(p, a);
+        else k_local_adamw<false, true><<<grid, kThreads, 0, s>>>(p, a);
+    } else {
+        if (p.grad_bf16) k_local_adamw<true, false><<<grid, kThreads, 0, s>>>(p, a);
+        else k_local_adamw<false, false><<<grid, kThreads, 0, s>>>(p, a);
+    }
     return cudaGetLastError();
 }
 
-cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, cudaStream_t s) {
-    const int grid = clamp_grid(ls.grid_sgdm, static_cast<uint64_t>(p.num_tiles) * p.n);
+cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, bool from_x,
+                              cudaStream_t s) {
+    const uint64_t items = static_cast<uint64_t>(p.num_tiles) * p.n;
+    const int grid = clamp_grid(from_x ? ls.grid_sgdm_from_x : ls.grid_sgdm, items);
     if (grid == 0) return cudaSuccess;
-    if (p.grad_bf16) k_local_sgdm<true><<<grid, kThreads, 0, s>>>(p, a);
-    else k_local_sgdm<false><<<grid, kThreads, 0, s>>>(p, a);
+    if (from_x) {
+        if (p.grad_bf16) k_local_sgdm<true, true><<<grid, kThreads, 0, s>>>(p, a);
+        else k_local_sgdm<false, true><<<grid, kThreads, 0, s>>>(p, a);
+    } else {
+        if (p.grad_bf16) k_local_sgdm<true, false><<<grid, kThreads, 0, s>>>(p, a);
+        else k_local_sgdm<false, false><<<grid, kThreads, 0, s>>>(p, a);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
+                                     const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s) {
+    if (!fused_round_available(p)) return cudaErrorInvalidValue;
+    const int grid = clamp_grid(ls.grid_fused, p.num_tiles);
+    if (grid == 0) return cudaSuccess;
+    fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, kFusedSmem, s>>>(p, a, sa, g, from_x ? 1 : 0);
     return cudaGetLastError();
 }
 

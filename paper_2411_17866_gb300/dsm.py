@@ -24,6 +24,7 @@ SIGN, RSIGN_ZERO, RSIGN_PM = 0, 1, 2
 F32, BF16 = 0, 1
 BUF_X, BUF_M, BUF_REPLICA, BUF_OPT_M, BUF_OPT_V, BUF_GRAD, BUF_GLOBAL_V = 0, 1, 2, 3, 4, 5, 6
 GLOBAL_SIGN_MOMENTUM, GLOBAL_SLOWMO, GLOBAL_SIGNED_SLOWMO, GLOBAL_LOOKAHEAD, GLOBAL_ADAMW = 0, 1, 2, 3, 4
+FLAG_FUSED_ROUND = 1
 
 ERROR_NAMES = {DSM_EINVAL: "DSM_EINVAL", DSM_ENOMEM: "DSM_ENOMEM", DSM_EALIGN: "DSM_EALIGN",
                DSM_ESTATE: "DSM_ESTATE", DSM_ECUDA: "DSM_ECUDA", DSM_ERANGE: "DSM_ERANGE"}
@@ -48,7 +49,7 @@ class dsm_hparams(ctypes.Structure):
     _fields_ = [("base", c_int32), ("lr", c_float), ("b1", c_float), ("b2", c_float), ("eps", c_float),
                 ("wd", c_float), ("mu", c_float), ("g_b1", c_float), ("g_b2", c_float), ("g_eta", c_float),
                 ("g_wd", c_float), ("sign_mode", c_int32), ("rsign_B", c_float), ("grad_dtype", c_int32),
-                ("reserved", c_uint32), ("seed", c_uint64), ("global_mode", c_int32), ("g_eps", c_float)]
+                ("flags", c_uint32), ("seed", c_uint64), ("global_mode", c_int32), ("g_eps", c_float)]
 
 
 class dsm_tensor_stats(ctypes.Structure):
@@ -144,14 +145,9 @@ def make_layout(tensors):
 def make_hparams(hp) -> dsm_hparams:
     """A dsm_hparams from an object with the same field names."""
     h = dsm_hparams()
+    defaults = {"global_mode": 0, "g_eps": 1e-8, "flags": 0}
     for name, _ in dsm_hparams._fields_:
-        if name == "reserved":
-            continue
-        if name in ("global_mode", "g_eps") and not hasattr(hp, name):
-            setattr(h, name, 0 if name == "global_mode" else 1e-8)
-            continue
-        setattr(h, name, getattr(hp, name))
-    h.reserved = 0
+        setattr(h, name, getattr(hp, name, defaults.get(name)))
     return h
 
 

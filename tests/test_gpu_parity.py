@@ -108,6 +108,59 @@ def test_global_variants_bitexact(layout_name, name, hp, n, tau):
     run.close()
 
 
+FUSED = [
+    ("adamw-f32-n4-t3", ADAMW, 4, 3),
+    ("adamw-bf16-n8-t2", dataclasses.replace(ADAMW, grad_dtype=W.BF16), 8, 2),
+    ("sgdm-rsign-n8-t1", SGDM, 8, 1),
+    ("sgdm-rsignpm-n3-t2", dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, grad_dtype=W.BF16), 3, 2),
+    ("adamw-n1-t1", ADAMW, 1, 1),
+    ("adamw-n5-t2", ADAMW, 5, 2),
+    ("adamw-n9-unfused", ADAMW, 9, 2),
+    ("slowmo-unfused", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO), 4, 2),
+]
+
+
+@pytest.mark.parametrize("layout_name", ["ragged", "mini"])
+@pytest.mark.parametrize("name,hp,n,tau", FUSED, ids=[c[0] for c in FUSED])
+def test_fused_round_bitexact(layout_name, name, hp, n, tau):
+    """The fused round (last local step inside the global step, lazy reset) gives the same state."""
+    tensors = RAGGED if layout_name == "ragged" else MINI
+    hp = dataclasses.replace(hp, flags=W.FLAG_FUSED_ROUND)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    for _ in range(3):
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+        compare_state(run, ora)      # replicas read while their reset is pending return x
+        compare_stats(stats, ora.last_stats, n)
+    run.close()
+
+
+def test_fused_round_pending_step_is_materialized():
+    """Reading worker state while the last local step is deferred runs that step first."""
+    tensors, n, tau = MINI, 4, 2
+    hp = dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp)
+    for t in range(3):
+        for k in range(tau):
+            run.fill_synthetic_grads(t * tau + k)
+            run.local_step()
+            ora.local_step()
+        if t == 1:   # deferred step: reading a replica runs it unfused, then the global step is unfused
+            assert_bitexact(run.read(dsm.BUF_REPLICA, 2).numpy(), ora.X[2], "replica before global step")
+        if t == 2:   # writing replicas while their reset is pending writes x into them first
+            run.global_step()
+            ora.global_step()
+            run.write(dsm.BUF_REPLICA, torch.from_numpy(ora.X[1].copy()), worker=1)
+            compare_state(run, ora)
+            continue
+        run.global_step()
+        ora.global_step()
+        compare_state(run, ora)
+    run.close()
+
+
 def test_caller_gradients_host_and_device():
     """dsm_load_grads: gradients written by the caller (pinned host and device)."""
     tensors, n, tau = MINI, 3, 2
@@ -210,15 +263,17 @@ def test_x0_from_device_and_host():
         run.close()
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
 @pytest.mark.parametrize("key", list(W.WORKLOADS))
-def test_full_workloads_sampled(key):
+def test_full_workloads_sampled(key, fused):
     """Each measured workload at full size, one round, in the launch sequence the benchmark uses,
     checked on sampled elements against the element-subset oracle (first and last 64 elements of
     every tensor plus 20000 random ones; the whole model for the flat workload)."""
     wl = W.WORKLOADS[key]
-    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, wl.hp)
+    hp = dataclasses.replace(wl.hp, flags=W.FLAG_FUSED_ROUND if fused else 0)
+    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp)
     elems = None if wl.d <= (1 << 20) else sample_elements(wl.tensors, 20000)
-    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=elems, with_stats=elems is None)
+    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, hp, elems=elems, with_stats=elems is None)
     rounds = wl.rounds if elems is None else 1
     for _ in range(rounds):
         stats = run.synthetic_round(with_stats=True)

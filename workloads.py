@@ -41,6 +41,8 @@ GLOBAL_SLOWMO = 1
 GLOBAL_SIGNED_SLOWMO = 2
 GLOBAL_LOOKAHEAD = 3
 GLOBAL_ADAMW = 4
+# Execution flags
+FLAG_FUSED_ROUND = 1
 
 VOCAB = 50257
 CONTEXT = 1024
@@ -74,6 +76,7 @@ class HParams:
     seed: int = 0
     global_mode: int = 0      # GLOBAL_* below
     g_eps: float = 1e-8       # epsilon of the global AdamW step
+    flags: int = 0            # FLAG_* below (execution options; the results do not depend on them)
 
 
 @dataclasses.dataclass(frozen=True)
