@@ -278,6 +278,12 @@ int dsm_set_round(dsm_handle* h, uint64_t round);
 
 int dsm_get_info(const dsm_handle* h, dsm_info* out);
 
+/* Memory-safety check (no counterpart in the paper): every buffer of the
+ * arena is followed by a 256-byte guard region filled with 0xA5 at create;
+ * a write past the end of any buffer changes it.  Synchronises the stream
+ * and sets *bad_regions to the number of guard regions that changed. */
+int dsm_check_guards(dsm_handle* h, dsm_stream_t stream, uint32_t* bad_regions);
+
 /* Release the handle's host metadata; the arena stays the caller's.
  * NULL is accepted. */
 int dsm_destroy(dsm_handle* h);

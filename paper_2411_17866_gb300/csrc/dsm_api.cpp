@@ -37,6 +37,8 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 constexpr uint64_t kAlign = 256;
+constexpr uint64_t kGuardBytes = 256;       // guard region after every arena buffer
+constexpr unsigned char kGuardByte = 0xA5;  // its fill pattern
 constexpr uint64_t kStrideAlign = 64;  // elements; keeps every worker slice 256-byte aligned
 constexpr uint64_t kMaxD = 1ull << 40;
 
@@ -65,6 +67,7 @@ struct ArenaLayout {
     uint64_t off_tensors = 0, off_tiles = 0, off_x = 0, off_m = 0, off_gv = 0, off_X = 0, off_om = 0, off_ov = 0,
              off_grad = 0, off_partials = 0, off_stats = 0, total = 0;
     size_t grad_esize = 4;
+    std::vector<uint64_t> guards;  // offsets of the guard regions
 };
 
 int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp, ArenaLayout* al) {
@@ -124,9 +127,11 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
     a.num_tiles = static_cast<uint32_t>(tiles);
     a.grad_esize = hp->grad_dtype == DSM_BF16 ? 2 : 4;
     uint64_t off = 0;
-    auto take = [&](uint64_t bytes) {
+    auto take = [&](uint64_t bytes) {  // a buffer, then its guard region
         const uint64_t o = off;
         off = round_up(off + bytes, kAlign);
+        a.guards.push_back(off);
+        off += kGuardBytes;
         return o;
     };
     a.off_tensors = take(uint64_t(a.num_tensors) * sizeof(TensorDesc));
@@ -397,6 +402,8 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     const uint64_t zero_from = al.off_m;
     if ((err = cudaMemsetAsync(A + zero_from, 0, al.total - zero_from, s)) != cudaSuccess)
         return bail(err, "zero the state");
+    for (uint64_t g : al.guards)
+        if ((err = cudaMemsetAsync(A + g, kGuardByte, kGuardBytes, s)) != cudaSuccess) return bail(err, "fill guards");
     if (x0) {
         if ((err = cudaMemcpyAsync(p.x, x0, al.d * 4, x0_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice,
                                    s)) != cudaSuccess)
@@ -628,6 +635,30 @@ int dsm_set_round(dsm_handle* h, uint64_t round) {
     }
     h->gb1_pow = q1;
     h->gb2_pow = q2;
+    return DSM_OK;
+}
+
+int dsm_check_guards(dsm_handle* h, dsm_stream_t stream, uint32_t* bad_regions) {
+    if (!h || !bad_regions) return fail(DSM_EINVAL, "NULL argument");
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    std::vector<unsigned char> buf(h->al.guards.size() * kGuardBytes);
+    cudaStream_t s = S(stream);
+    cudaError_t err;
+    for (size_t i = 0; i < h->al.guards.size(); ++i)
+        if ((err = cudaMemcpyAsync(buf.data() + i * kGuardBytes, h->arena + h->al.guards[i], kGuardBytes,
+                                   cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return cuda_fail(err, "read guards");
+    if ((err = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(err, "synchronise after reading guards");
+    uint32_t bad = 0;
+    for (size_t i = 0; i < h->al.guards.size(); ++i) {
+        for (uint64_t b = 0; b < kGuardBytes; ++b)
+            if (buf[i * kGuardBytes + b] != kGuardByte) {
+                ++bad;
+                break;
+            }
+    }
+    *bad_regions = bad;
     return DSM_OK;
 }
 

@@ -82,6 +82,7 @@ _PROTOS = {
     "dsm_set_round": (c_int, [c_void_p, c_uint64]),
     "dsm_cosine_gamma": (c_int, [c_float, c_float, c_uint64, c_uint64, c_uint64, POINTER(c_float)]),
     "dsm_get_info": (c_int, [c_void_p, POINTER(dsm_info)]),
+    "dsm_check_guards": (c_int, [c_void_p, c_void_p, POINTER(c_uint32)]),
     "dsm_destroy": (c_int, [c_void_p]),
     "dsm_last_error": (c_char_p, []),
     "dsm_global_step_noalloc": (c_int, [POINTER(dsm_layout), c_uint32, POINTER(dsm_hparams), c_float, c_uint64,
@@ -238,6 +239,13 @@ def dsm_get_info(h) -> dsm_info:
     return info
 
 
+def dsm_check_guards(h, stream=None) -> int:
+    """Number of arena guard regions that a write past the end of a buffer changed (0 = intact)."""
+    bad = c_uint32()
+    _check(load_library().dsm_check_guards(h, _stream(stream), byref(bad)), "dsm_check_guards")
+    return bad.value
+
+
 def dsm_destroy(h) -> None:
     _check(load_library().dsm_destroy(h), "dsm_destroy")
 
@@ -340,6 +348,9 @@ class DistributedSignMomentum:
 
     def info(self):
         return dsm_get_info(self.h)
+
+    def check_guards(self, stream=None) -> int:
+        return dsm_check_guards(self.h, stream)
 
     def close(self):
         if getattr(self, "h", None) is not None:

@@ -35,8 +35,10 @@ def assert_bitexact(got, want, what):
 
 
 def compare_state(run, ora, elems=None, grads=True):
-    """Every buffer of the GPU state against the oracle, bit for bit (optionally on a subset)."""
+    """Every buffer of the GPU state against the oracle, bit for bit (optionally on a subset);
+    also checks that no kernel wrote past the end of an arena buffer."""
     import torch
+    assert run.check_guards() == 0, "an arena guard region was overwritten"
     sel = slice(None) if elems is None else elems
 
     def rd(which, w=0):

@@ -326,3 +326,57 @@ def test_fp64_twin_within_stated_tolerance():
         diverged |= moved
     print(f"sign mismatches vs fp64: {mismatches} of {elems.size}")
     run.close()
+
+
+DEGENERATE = [
+    ("eta-zero", dataclasses.replace(ADAMW, g_eta=0.0), 3, 2),
+    ("global-betas-one", dataclasses.replace(ADAMW, g_b1=1.0, g_b2=1.0), 2, 2),
+    ("zero-global-decay-and-betas", dataclasses.replace(SGDM, sign_mode=W.SIGN, g_b1=0.0, g_b2=0.0, g_wd=0.0), 4, 1),
+    ("rsign-huge-bound", dataclasses.replace(SGDM, rsign_B=1e30), 3, 1),
+    ("rsign-tiny-bound", dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, rsign_B=1e-30), 3, 1),
+    ("tiny-gamma", dataclasses.replace(ADAMW, lr=1e-8), 2, 3),
+    ("large-seed-tau5", dataclasses.replace(ADAMW, seed=(1 << 63) + 5), 2, 5),
+    ("max-workers-64", dataclasses.replace(SGDM, seed=3), 64, 1),
+]
+
+
+@pytest.mark.parametrize("name,hp,n,tau", DEGENERATE, ids=[c[0] for c in DEGENERATE])
+def test_degenerate_cases_bitexact(name, hp, n, tau):
+    """Degenerate settings of the method and the maximum worker count, against the oracle."""
+    tensors = RAGGED
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    for _ in range(2):
+        x_before = ora.x.copy()
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+        compare_state(run, ora)
+        compare_stats(stats, ora.last_stats, n)
+        if name == "eta-zero":
+            assert np.array_equal(ora.x, x_before)
+        if name == "rsign-tiny-bound":   # every nonzero u is above the bound: deterministic sign, all counted
+            nonzero = int(np.count_nonzero(ora.last_inter["u"]))
+            assert sum(s["clamped"] for s in stats) == nonzero
+    run.close()
+
+
+def test_zero_gradients():
+    """All-zero gradients (scale 0): the workers only decay; Delta = lr * lambda * x for AdamW."""
+    tensors = tuple(dataclasses.replace(t, grad_scale=0.0) for t in RAGGED)
+    run = dsm.DistributedSignMomentum(tensors, 3, 2, ADAMW)
+    ora = O.OracleRun(tensors, 3, 2, ADAMW, with_stats=True)
+    run.synthetic_round()
+    ora.run_round()
+    compare_state(run, ora)
+    run.close()
+
+
+def test_guard_regions_detect_an_overrun():
+    """A byte written past the end of the tensor table (a planted host-side write) is reported."""
+    run = dsm.DistributedSignMomentum(MINI, 2, 1, ADAMW)
+    assert run.check_guards() == 0
+    first_guard = -(-len(MINI) * 48 // 256) * 256
+    run.arena[first_guard + 7] = 0
+    torch.cuda.synchronize()
+    assert run.check_guards() == 1
+    run.close()
