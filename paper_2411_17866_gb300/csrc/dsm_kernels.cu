@@ -559,6 +559,85 @@ __device__ __forceinline__ void global_elem_generic(const Problem& p, const Glob
     for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = x;
 }
 
+// Global step on a thread's 4 aligned elements for any number of workers:
+// 16-byte accesses, the replicas read once for the average and once more
+// (from L2) for the statistics, then overwritten by the reset.
+template <int MODE>
+__device__ __forceinline__ void global_vec_generic(const Problem& p, const GlobalScalars& g, float lam,
+                                                   uint64_t gi, ThreadStats& st) {
+    float x[4], m[4], v[4] = {0.f, 0.f, 0.f, 0.f}, acc[4] = {0.f, 0.f, 0.f, 0.f};
+    load4(p.x + gi, x);
+    load4(p.m + gi, m);
+    if (MODE == 4) load4(p.gv + gi, v);
+    // pass 1: the average; the loads of up to kGenChunk workers are issued before their additions,
+    // which stay in worker order (kept in L2 for pass 2)
+    constexpr uint32_t kGenChunk = 8;
+    for (uint32_t i0 = 0; i0 < p.n; i0 += kGenChunk) {
+        float4 r[kGenChunk];
+#pragma unroll
+        for (uint32_t c = 0; c < kGenChunk; ++c)
+            if (i0 + c < p.n) r[c] = *reinterpret_cast<const float4*>(p.X + (i0 + c) * p.d_stride + gi);
+#pragma unroll
+        for (uint32_t c = 0; c < kGenChunk; ++c) {
+            if (i0 + c < p.n) {
+                acc[0] = __fadd_rn(acc[0], __fsub_rn(x[0], r[c].x));
+                acc[1] = __fadd_rn(acc[1], __fsub_rn(x[1], r[c].y));
+                acc[2] = __fadd_rn(acc[2], __fsub_rn(x[2], r[c].z));
+                acc[3] = __fadd_rn(acc[3], __fsub_rn(x[3], r[c].w));
+            }
+        }
+    }
+    float ru[4] = {0.f, 0.f, 0.f, 0.f};
+    if (MODE == 0 && g.sign_mode != 0) {
+        const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+        ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
+    }
+    float D[4], xn[4], dr[4] = {0.f, 0.f, 0.f, 0.f};
+    int sD[4];
+    bool unan[4] = {true, true, true, true};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        D[j] = __fdiv_rn(acc[j], g.n_f);
+        sD[j] = sgn(D[j]);
+        xn[j] = x[j];
+        float u, s;
+        global_update<MODE>(D[j], xn[j], m[j], v[j], g, lam, ru[j], u, s);
+        st.zero += (s == 0.f);
+        st.flips += (sgn(u) != sD[j]);
+        st.clamped += (MODE == 0 && g.sign_mode != 0 && fabsf(u) > g.B);
+        csum_add(st.dsq, __fmul_rn(D[j], D[j]));
+    }
+    // pass 2: the statistics and the reset, again kGenChunk workers' loads at a time
+    for (uint32_t i0 = 0; i0 < p.n; i0 += kGenChunk) {
+        float4 r[kGenChunk];
+#pragma unroll
+        for (uint32_t c = 0; c < kGenChunk; ++c)
+            if (i0 + c < p.n) r[c] = __ldcs(reinterpret_cast<const float4*>(p.X + (i0 + c) * p.d_stride + gi));
+#pragma unroll
+        for (uint32_t c = 0; c < kGenChunk; ++c) {
+            if (i0 + c < p.n) {
+                const float rr[4] = {r[c].x, r[c].y, r[c].z, r[c].w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float di = __fsub_rn(x[j], rr[j]);
+                    const float ei = __fsub_rn(di, D[j]);
+                    dr[j] = __fadd_rn(dr[j], __fmul_rn(ei, ei));
+                    unan[j] = unan[j] && (sgn(di) == sD[j]);
+                }
+                store4(p.X + (i0 + c) * p.d_stride + gi, xn);
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        csum_add(st.drift, dr[j]);
+        st.unanimous += unan[j];
+    }
+    store4(p.x + gi, xn);
+    store4(p.m + gi, m);
+    if (MODE == 4) store4(p.gv + gi, v);
+}
+
 // K4: the fused global step (average over the replicas, sign-momentum update,
 // momentum update, reset of every replica) with statistics.
 // NW > 0: exactly NW replicas, held in registers and double-buffered.
@@ -628,6 +707,8 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
             if (MODE == 4) store4(p.gv + gi, cv);
 #pragma unroll
             for (int i = 0; i < W; ++i) store4(p.X + i * p.d_stride + gi, cx);
+        } else if (NW == 0 && vector_ok(td, e0)) {
+            global_vec_generic<MODE>(p, g, lam, td.start + e0, st);
         } else {
             const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
             for (uint32_t e = e0; e < e1; ++e) global_elem_generic<MODE>(p, g, lam, td.start + e, st);
