@@ -746,13 +746,19 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // A CTA walks its tiles worker by worker; each thread keeps the next
 // kFusedDepth (tile, worker) items in flight with cp.async into its own
 // shared-memory slots (x_i, m_i, v_i, g_i, and x, m with a tile's first worker).
-constexpr int kFusedDepth = 3;
+// Items in flight per thread: 2, or 3 for AdamW with more than 4 workers,
+// whose registers already limit the resident CTAs (measured on GB300: depth 2
+// gives 0.92 / 1.00 of the copy bandwidth on GPT-2 S (AdamW, n = 4) / L
+// (SGD-momentum, n = 8), depth 3 gives 0.85 on GPT-2 M (AdamW, n = 8) where
+// depth 2 gives 0.79).
 constexpr int kFusedStreams = 6;
-constexpr size_t kFusedSmem = size_t(kFusedDepth) * kFusedStreams * kThreads * sizeof(float4);
+__host__ __device__ constexpr int fused_depth(bool adamw, int nw) { return (adamw && nw > 4) ? 3 : 2; }
+__host__ __device__ constexpr size_t fused_smem(int depth) { return size_t(depth) * kFusedStreams * kThreads * sizeof(float4); }
 
 template <bool kAdamW, bool kBf16, int NW>
 __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
                                                                 GlobalScalars g, int from_global) {
+    constexpr int kFusedDepth = fused_depth(kAdamW, NW);
     extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     auto slot = [&](int it, int stream) -> float4* {
@@ -979,6 +985,8 @@ FusedKernel fused_kernel_for(const Problem& p, bool adamw) {
     return p.grad_bf16 ? fused_kernel_n<false, true>(p.n) : fused_kernel_n<false, false>(p.n);
 }
 
+size_t fused_smem_for(const Problem& p, bool adamw) { return fused_smem(fused_depth(adamw, int(p.n))); }
+
 }  // namespace
 
 bool fused_round_available(const Problem& p) {
@@ -999,9 +1007,10 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     out->grid_sgdm = p.grad_bf16 ? grid_for(k_local_sgdm<true, false>, sms) : grid_for(k_local_sgdm<false, false>, sms);
     if (fused_round_available(p)) {
         const FusedKernel fk = fused_kernel_for(p, p.opt_v != nullptr);
-        cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kFusedSmem));
+        const size_t smem = fused_smem_for(p, p.opt_v != nullptr);
+        cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         if (e != cudaSuccess) return e;
-        out->grid_fused = grid_for(fk, sms, kFusedSmem);
+        out->grid_fused = grid_for(fk, sms, smem);
         out->grid_adamw_from_x = p.grad_bf16 ? grid_for(k_local_adamw<true, true>, sms) : grid_for(k_local_adamw<false, true>, sms);
         out->grid_sgdm_from_x = p.grad_bf16 ? grid_for(k_local_sgdm<true, true>, sms) : grid_for(k_local_sgdm<false, true>, sms);
     }
@@ -1064,7 +1073,8 @@ cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, co
     if (!fused_round_available(p)) return cudaErrorInvalidValue;
     const int grid = clamp_grid(ls.grid_fused, p.num_tiles);
     if (grid == 0) return cudaSuccess;
-    fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, kFusedSmem, s>>>(p, a, sa, g, from_x ? 1 : 0);
+    fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, fused_smem_for(p, p.opt_v != nullptr), s>>>(
+        p, a, sa, g, from_x ? 1 : 0);
     return cudaGetLastError();
 }
 
