@@ -402,9 +402,6 @@ def global_step_adamw(x, m, v, X, gamma, t: int, b1, b2, eps, eta, lam_e, dt):
     return x_new, m_new, v_new, {"delta": delta, "u": m_new, "sg": sign(m_new), "diffs": diffs}
 
 
-STAT_FIELDS = ("delta_sq", "drift", "zero_sign", "flips", "unanimous", "clamped")
-
-
 def round_stats(inter, tensor_of, num_tensors: int, sign_mode: int, B) -> list:
     """Per-tensor statistics of one global step, accumulated in float64 in element order.
 

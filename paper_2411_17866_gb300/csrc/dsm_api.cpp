@@ -232,11 +232,9 @@ int resolve_buffer(dsm_handle* h, int which, uint32_t worker, uint64_t offset, u
     return DSM_OK;
 }
 
-int copy_kind(const void* host_or_dev, int is_device, bool to_device, cudaMemcpyKind* kind) {
-    (void)host_or_dev;
-    if (to_device) *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
-    else *kind = is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
-    return DSM_OK;
+cudaMemcpyKind copy_kind(int other_is_device, bool to_device) {
+    if (other_is_device) return cudaMemcpyDeviceToDevice;
+    return to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost;
 }
 
 // Scalars of the next local step (count j + 1); advances the beta powers.
@@ -565,8 +563,7 @@ int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64
         if (rc != DSM_OK) return rc;
     }
     if (which == DSM_BUF_REPLICA && h->replicas_stale) src = reinterpret_cast<char*>(h->prob.x + offset);
-    cudaMemcpyKind kind;
-    copy_kind(dst, dst_is_device, false, &kind);
+    const cudaMemcpyKind kind = copy_kind(dst_is_device, false);
     cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "read buffer");
     if (!dst_is_device && (err = cudaStreamSynchronize(S(stream))) != cudaSuccess)
@@ -586,8 +583,7 @@ int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src,
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     if ((rc = materialize_pending(h, S(stream))) != DSM_OK) return rc;
     if ((rc = materialize_replicas(h, S(stream))) != DSM_OK) return rc;
-    cudaMemcpyKind kind;
-    copy_kind(src, src_is_device, true, &kind);
+    const cudaMemcpyKind kind = copy_kind(src_is_device, true);
     cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "write buffer");
     if (!src_is_device && (err = cudaStreamSynchronize(S(stream))) != cudaSuccess)

@@ -153,7 +153,3 @@ WORKLOADS = {
 # The workload the throughput line is quoted on.
 BENCH_WORKLOAD = "gpt2s"
 
-
-def init_value_kind(kind: int) -> str:
-    """How a tensor kind is initialised: 'hash' (0.02*(2u-1)), 'one' or 'zero'."""
-    return {KIND_WEIGHT: "hash", KIND_LN_W: "one"}.get(kind, "zero")
