@@ -321,9 +321,17 @@ def main():
     local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
     local_bytes_from_x = wl.n * wl.d * (bytes_per_elem_local(wl) - 4) + wl.d * 4
 
-    def round_(t, local_events=None, global_events=None):
+    def round_(t, local_events=None, global_events=None, fill_events=None):
         for k in range(tau):
-            run.fill_synthetic_grads(t * tau + k, stream)
+            if fill_events is not None:
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                run.fill_synthetic_grads(t * tau + k, stream)
+                b.record(stream)
+                fill_events.append((a, b))
+            else:
+                run.fill_synthetic_grads(t * tau + k, stream)
             if local_events is not None and not (fused and k == tau - 1):
                 a = torch.cuda.Event(enable_timing=True)
                 b = torch.cuda.Event(enable_timing=True)
@@ -354,7 +362,7 @@ def main():
     sampler = ClockSampler(local) if (rank == 0 and not args.no_clocks) else None
     if sampler:
         sampler.start()
-    local_ev, global_ev = [], []
+    local_ev, global_ev, fill_ev = [], [], []
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -362,7 +370,7 @@ def main():
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for _ in range(args.steps):
-        round_(t, local_ev, global_ev)
+        round_(t, local_ev, global_ev, fill_ev)
         t += 1
     end.record(stream)
     torch.cuda.synchronize()
@@ -373,6 +381,7 @@ def main():
     local_ms = [a.elapsed_time(b) for a, b, _ in local_ev]
     local_launch_bytes = [nb for _, _, nb in local_ev]
     global_ms = [a.elapsed_time(b) for a, b in global_ev]
+    fill_ms = [a.elapsed_time(b) for a, b in fill_ev]
 
     # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device
     # gradient copy + local step), the global step, and the new x read back to pinned host memory
@@ -411,6 +420,7 @@ def main():
     # fused round: the last local step runs inside the global-step launch
     global_bytes = wl.d * (bytes_per_param_global(wl) if not fused else bytes_per_param_fused_last(wl))
     avg_local_s = statistics.mean(local_ms) / 1e3
+    grad_bytes = wl.n * wl.d * (2 if wl.hp.grad_dtype == W.BF16 else 4)
     achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
     kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
     traffic = committed_traffic(f"{kname}:{args.workload}")
@@ -431,6 +441,10 @@ def main():
                         "note": ("last local step fused with the global step, + statistics reduction"
                                  if fused else "fused global step + statistics reduction") +
                                 ", CUDA events around both"},
+        "grad_fill": {"avg_ms": statistics.mean(fill_ms), "bytes_written_per_launch": grad_bytes,
+                      "write_gbs": grad_bytes / (statistics.mean(fill_ms) / 1e3) / 1e9,
+                      "note": "synthetic gradients (stand-in for the backward pass); bound by instruction "
+                              "issue of the SplitMix64 hash"},
         "optimizer_only_value": wl.d * args.steps / ((sum(local_ms) + sum(global_ms)) / 1e3),
         "gpu_launches": args.steps * (2 * tau + (1 if fused else 2)),
         "e2e": e2e,

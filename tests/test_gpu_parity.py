@@ -387,3 +387,21 @@ def test_guard_regions_detect_an_overrun():
     torch.cuda.synchronize()
     assert run.check_guards() == 1
     run.close()
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+def test_many_rounds_stay_bitexact(fused):
+    """Forty rounds with a learning-rate schedule: no drift between the GPU and the oracle."""
+    tensors, n, tau = RAGGED, 3, 2
+    hp = dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND if fused else 0, sign_mode=W.SIGN)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    for t in range(40):
+        gamma = dsm.dsm_cosine_gamma(6e-4, 0.05, 10, 80, t * tau)
+        run.set_gamma(gamma)
+        ora.gamma = float(gamma)
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+        compare_stats(stats, ora.last_stats, n)
+    compare_state(run, ora)
+    run.close()
