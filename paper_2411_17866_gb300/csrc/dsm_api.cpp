@@ -7,6 +7,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -320,7 +321,9 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
         return fail(DSM_EALIGN, "arena %p is not device memory", dev_arena);
 
-    dsm_handle* h = new (std::nothrow) dsm_handle();
+    // DSM_INJECT_HOST_ALLOC_FAILURE=1 makes this allocation fail (host-side fault injection for tests)
+    const char* inject = std::getenv("DSM_INJECT_HOST_ALLOC_FAILURE");
+    dsm_handle* h = (inject && inject[0] == '1') ? nullptr : new (std::nothrow) dsm_handle();
     if (!h) return fail(DSM_ENOMEM, "out of host memory for the handle");
     h->device = attr.device;
     h->n = n;

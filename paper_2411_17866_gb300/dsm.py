@@ -352,6 +352,35 @@ class DistributedSignMomentum:
     def check_guards(self, stream=None) -> int:
         return dsm_check_guards(self.h, stream)
 
+    def state_dict(self) -> dict:
+        """Every buffer of the method's state as CPU tensors, with the round counter and gamma_t
+        (call between rounds).  Gradients are not part of the state."""
+        info = dsm_get_info(self.h)
+        if info.local_steps != 0:
+            raise DsmError(DSM_ESTATE, "state_dict", "take a checkpoint between rounds")
+        st = {"round": int(info.round), "gamma": float(info.gamma), "x": self.read(BUF_X), "m": self.read(BUF_M),
+              "replicas": [self.read(BUF_REPLICA, i) for i in range(self.n)],
+              "opt_m": [self.read(BUF_OPT_M, i) for i in range(self.n)]}
+        if self.hp.base == BASE_ADAMW:
+            st["opt_v"] = [self.read(BUF_OPT_V, i) for i in range(self.n)]
+        if self.hp.global_mode == GLOBAL_ADAMW:
+            st["global_v"] = self.read(BUF_GLOBAL_V)
+        return st
+
+    def load_state_dict(self, st: dict) -> None:
+        """Restore a state_dict() into this handle (same layout, n and hyper-parameters)."""
+        self.write(BUF_X, st["x"])
+        self.write(BUF_M, st["m"])
+        for i in range(self.n):
+            self.write(BUF_REPLICA, st["replicas"][i], worker=i)
+            self.write(BUF_OPT_M, st["opt_m"][i], worker=i)
+            if "opt_v" in st:
+                self.write(BUF_OPT_V, st["opt_v"][i], worker=i)
+        if "global_v" in st:
+            self.write(BUF_GLOBAL_V, st["global_v"])
+        dsm_set_round(self.h, st["round"])
+        dsm_set_gamma(self.h, st["gamma"])
+
     def close(self):
         if getattr(self, "h", None) is not None:
             dsm_destroy(self.h)

@@ -143,3 +143,18 @@ def test_cosine_schedule_matches_the_oracle(lib):
     for bad in [(0.0, r, W_, S, 0), (P, 1.5, W_, S, 0), (P, r, S + 1, S, 0), (P, r, 0, 0, 0)]:
         with pytest.raises(dsm.DsmError):
             dsm.dsm_cosine_gamma(*bad)
+
+
+def test_host_memory_arena_is_refused(lib):
+    """A host buffer as arena: DSM_EALIGN ('not device memory') with a GPU, DSM_ECUDA (the runtime's
+    message) without one; never a crash."""
+    lay, n, hp = _args()
+    need = dsm.dsm_state_bytes(lay, n, hp)
+    arena = ctypes.create_string_buffer(need + 256)
+    ptr = (ctypes.addressof(arena) + 255) // 256 * 256
+    h = ctypes.c_void_p()
+    rc = lib.dsm_create(ctypes.byref(lay), n, 2, ctypes.byref(hp), ctypes.c_void_p(ptr), need, None, 0, None,
+                        ctypes.byref(h))
+    assert rc in (dsm.DSM_ECUDA, dsm.DSM_EALIGN)
+    msg = dsm.last_error()
+    assert ("device memory" in msg) if rc == dsm.DSM_EALIGN else ("cudaPointerGetAttributes" in msg)

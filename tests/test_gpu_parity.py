@@ -405,3 +405,31 @@ def test_many_rounds_stay_bitexact(fused):
         compare_stats(stats, ora.last_stats, n)
     compare_state(run, ora)
     run.close()
+
+
+def test_injected_host_allocation_failure_on_device_arena(monkeypatch):
+    """With a valid device arena, the injected host allocation failure is reported as DSM_ENOMEM."""
+    monkeypatch.setenv("DSM_INJECT_HOST_ALLOC_FAILURE", "1")
+    with pytest.raises(dsm.DsmError) as e:
+        dsm.DistributedSignMomentum(MINI, 2, 1, ADAMW)
+    assert e.value.code == dsm.DSM_ENOMEM
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+def test_state_dict_round_trip(fused):
+    """Checkpoint after a round, restore into a fresh handle, continue: identical to never stopping."""
+    hp = dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND if fused else 0, global_mode=W.GLOBAL_SIGN_MOMENTUM)
+    a = dsm.DistributedSignMomentum(RAGGED, 3, 2, hp)
+    a.set_gamma(5e-4)
+    a.synthetic_round()
+    st = a.state_dict()
+    b = dsm.DistributedSignMomentum(RAGGED, 3, 2, hp, x0=torch.zeros(a.d))
+    b.load_state_dict(st)
+    for _ in range(2):
+        a.synthetic_round()
+        b.synthetic_round()
+    torch.cuda.synchronize()
+    for which, w in [(dsm.BUF_X, 0), (dsm.BUF_M, 0)] + [(dsm.BUF_OPT_V, i) for i in range(3)]:
+        assert torch.equal(a.read(which, w), b.read(which, w))
+    a.close()
+    b.close()
