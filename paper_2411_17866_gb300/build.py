@@ -45,22 +45,30 @@ def _run(cmd, verbose):
     return r.stdout
 
 
-def build(verbose: bool = False, extra_flags=()) -> str:
-    """Compile and link libdsm.so; returns its path."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, fmad: bool = False, out: str = LIB) -> str:
+    """Compile and link libdsm.so (to ``out``); returns its path.
+
+    fmad=True builds with nvcc's default multiply-add contraction; the method's
+    arithmetic is written with explicit round-to-nearest intrinsics, which are
+    never contracted, so both builds give identical results (a GPU test checks).
+    """
+    objdir = os.path.join(BUILD, "fmad" if fmad else "nofmad")
+    os.makedirs(objdir, exist_ok=True)
+    os.makedirs(os.path.dirname(os.path.abspath(out)), exist_ok=True)
     nv = nvcc()
+    flags = [f for f in NVCC_FLAGS if not (fmad and f == "--fmad=false")]
     objs = []
     cmds = []
     for src in SOURCES:
-        obj = os.path.join(BUILD, src + ".o")
+        obj = os.path.join(objdir, src + ".o")
         objs.append(obj)
-        cmds.append([nv, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj])
+        cmds.append([nv, *ARCH, *flags, "-c", os.path.join(CSRC, src), "-o", obj])
     with ThreadPoolExecutor(max_workers=len(cmds)) as ex:
         list(ex.map(lambda c: _run(c, verbose), cmds))
-    tmp = LIB + ".tmp"
+    tmp = out + ".tmp"
     _run([nv, *ARCH, "-shared", "-o", tmp, *objs, "-lcudart_static", "-lrt", "-ldl", "-lpthread"], verbose)
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, out)
+    return out
 
 
 if __name__ == "__main__":

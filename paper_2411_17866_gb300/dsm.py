@@ -15,7 +15,8 @@ import os
 from ctypes import POINTER, byref, c_char_p, c_float, c_int, c_int32, c_size_t, c_uint32, c_uint64, c_void_p
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libdsm.so")
+# The in-tree library; DSM_LIBRARY may name another build of it (e.g. the contracting release build).
+LIB_PATH = os.environ.get("DSM_LIBRARY") or os.path.join(_HERE, "libdsm.so")
 
 DSM_OK, DSM_EINVAL, DSM_ENOMEM, DSM_EALIGN, DSM_ESTATE, DSM_ECUDA, DSM_ERANGE = 0, -1, -2, -3, -4, -5, -6
 KIND_WEIGHT, KIND_BIAS, KIND_LN_W, KIND_LN_B = 0, 1, 2, 3
