@@ -188,8 +188,11 @@ typedef struct {
 
 typedef struct dsm_handle dsm_handle;
 
-/* Bytes of device memory the arena must hold for this problem; 0 if the
- * arguments are invalid (dsm_last_error() says why). */
+/* Bytes of device memory the arena must hold for the state of Algorithm 1
+ * (x_{t,0}, m_t, n replicas x^{(i)}, n base-optimizer states, n gradient
+ * buffers, tables and statistics) for this layout, n and hparams; 0 if the
+ * arguments are invalid (dsm_last_error() says why).  Host only: touches no
+ * GPU.  Errors are those of dsm_create's argument checks. */
 size_t dsm_state_bytes(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp);
 
 /* Create a handle over the caller's arena and initialise the state of
@@ -217,14 +220,20 @@ int dsm_set_gamma(dsm_handle* h, float gamma);
  * backward pass.  Asynchronous. */
 int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream);
 
-/* Device pointer to worker `worker`'s gradient buffer (d elements of the
- * gradient type; consecutive workers are d_stride elements apart), for a
- * caller that writes gradients itself. */
+/* Device pointer to worker `worker`'s gradient buffer, for a caller that
+ * writes the update directions' inputs itself (the stochastic gradients
+ * grad f_i(x^{(i)}, xi^{(i)}) of Eq. (base-sgd)).  The buffer holds d
+ * elements of the gradient type; consecutive workers are d_stride elements
+ * apart (dsm_get_info).  The pointer stays valid, and owned by the arena,
+ * until dsm_destroy.  DSM_EINVAL for NULL arguments, DSM_ERANGE for
+ * worker >= n. */
 int dsm_grad_ptr(dsm_handle* h, uint32_t worker, void** dev_ptr);
 
-/* Copy all workers' gradients from src, a dense [n][d] array of the
- * gradient type in host (src_is_device = 0; pinned memory makes it
- * asynchronous) or device memory, into the gradient buffers. */
+/* Copy all workers' gradients (the grad f_i of Eq. (base-sgd)) from src, a
+ * dense [n][d] array of the gradient type in host (src_is_device = 0;
+ * pinned memory makes it asynchronous) or device memory, into the gradient
+ * buffers.  src stays the caller's.  DSM_EINVAL for NULL arguments,
+ * DSM_ECUDA if the copy fails to enqueue. */
 int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream_t stream);
 
 /* Local step k of the current round on every worker, Eq. (local-steps):
@@ -246,18 +255,24 @@ int dsm_local_step(dsm_handle* h, dsm_stream_t stream);
 int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats, uint32_t stats_count);
 
 /* Device pointer to the per-tensor statistics of the last global step
- * (num_tensors entries), valid once that step has run on the stream. */
+ * (num_tensors dsm_tensor_stats in the arena; see that struct for the
+ * quantities of Algorithm 1 they measure), valid once that step has run on
+ * the stream and until the next one.  DSM_EINVAL for NULL arguments. */
 int dsm_stats_ptr(dsm_handle* h, const dsm_tensor_stats** dev_ptr);
 
-/* Copy elements [offset, offset+count) of buffer `which` (DSM_BUF_*) of
- * worker `worker` (ignored for X and M) to dst (host or device memory).
- * Elements are fp32 except DSM_BUF_GRAD, which has the gradient type.
- * With a host dst the call synchronises the stream before returning. */
+/* Copy elements [offset, offset+count) of a buffer of Algorithm 1's state
+ * (DSM_BUF_*: x_{t,0}, m_t, x^{(i)}, the base optimizer's state, gradients)
+ * of worker `worker` (ignored for X, M and GLOBAL_V) to dst (host or device
+ * memory, the caller's).  Elements are fp32 except DSM_BUF_GRAD, which has
+ * the gradient type.  With a host dst the call synchronises the stream
+ * before returning.  DSM_EINVAL for an unknown or absent buffer,
+ * DSM_ERANGE for worker >= n or a range outside [0, d). */
 int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64_t offset,
                     uint64_t count, int dst_is_device, dsm_stream_t stream);
 
 /* The reverse of dsm_read_params (checkpoint restore, or a caller-set
- * state).  With a host src the call synchronises the stream. */
+ * state of Algorithm 1).  With a host src the call synchronises the
+ * stream.  Same errors as dsm_read_params. */
 int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src, uint64_t offset,
                      uint64_t count, int src_is_device, dsm_stream_t stream);
 
@@ -273,9 +288,13 @@ int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src,
 int dsm_cosine_gamma(float peak, float final_ratio, uint64_t warmup_steps, uint64_t total_steps, uint64_t step,
                      float* gamma);
 
-/* Set the round counter t (checkpoint restore); only between rounds. */
+/* Set the round counter t of Algorithm 1 (checkpoint restore): it keys the
+ * randomized sign and fixes the AdamW step counts j = t*tau + k + 1 and the
+ * global AdamW count t + 1.  Only between rounds, else DSM_ESTATE. */
 int dsm_set_round(dsm_handle* h, uint64_t round);
 
+/* Describe the handle (sizes, t and k of Algorithm 1, gamma_t) into *out.
+ * Host only.  DSM_EINVAL for NULL arguments. */
 int dsm_get_info(const dsm_handle* h, dsm_info* out);
 
 /* Memory-safety check (no counterpart in the paper): every buffer of the
@@ -284,11 +303,14 @@ int dsm_get_info(const dsm_handle* h, dsm_info* out);
  * and sets *bad_regions to the number of guard regions that changed. */
 int dsm_check_guards(dsm_handle* h, dsm_stream_t stream, uint32_t* bad_regions);
 
-/* Release the handle's host metadata; the arena stays the caller's.
- * NULL is accepted. */
+/* Release the handle's host metadata; the arena stays the caller's and may
+ * be freed once the stream's work on it is complete.  NULL is accepted.
+ * Infrastructure: no counterpart in the paper. */
 int dsm_destroy(dsm_handle* h);
 
-/* Message for the calling thread's last failed call ("" if none). */
+/* Message for the calling thread's last failed call ("" if none); the
+ * string is the library's and stays valid until that thread's next failing
+ * call.  Infrastructure: no counterpart in the paper. */
 const char* dsm_last_error(void);
 
 /* ---- global step without any device allocation ----------------------- */
