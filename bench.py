@@ -264,7 +264,11 @@ def run_reference(args):
     import numpy as np
 
     from oracle import dsm_oracle as O
-    count = min(1 << 20, wl.d)
+    # each step one round over a contiguous sample, sized so that the whole run stays near a minute of
+    # CPU time whatever --steps and --warmup are (about 2^20 elements per step at the defaults)
+    per_step = (1 << 20) * (20 + 3) // max(1, args.steps + args.warmup)
+    per_step = per_step * 48 // (wl.n * wl.tau)          # the defaults' n*tau is 48
+    count = int(min(max(per_step, 1 << 14), 1 << 22, wl.d))
     ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64))
     for _ in range(args.warmup):
         ora.run_round()
