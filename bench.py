@@ -40,7 +40,16 @@ import workloads as W  # noqa: E402
 METRIC = "params/s per global round (τ local + sign-momentum step); % HBM roofline"
 UNIT = "params/s"
 CPU_SAMPLE_ELEMS = 1 << 22
-KERNELS_SRC = os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", "dsm_kernels.cu")
+# the sources of the local-step kernels (their arithmetic lives in the shared device header)
+KERNELS_SRC = [os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", f) for f in ("dsm_device.cuh", "dsm_kernels.cu")]
+
+
+def kernels_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNELS_SRC:
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 def parse():
@@ -150,8 +159,8 @@ def bytes_per_param_global(wl) -> int:
 
 
 def fused_round_active(wl) -> bool:
-    """The library fuses the round for the sign-momentum global step with n <= 8."""
-    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.hp.global_mode == W.GLOBAL_SIGN_MOMENTUM and wl.n <= 8
+    """The library fuses the round for every global step but global AdamW, with n <= 8."""
+    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.hp.global_mode != W.GLOBAL_ADAMW and wl.n <= 8
 
 
 def bytes_per_param_fused_last(wl) -> int:
@@ -178,9 +187,8 @@ def committed_traffic(kernel_key):
         return None
     with open(p) as f:
         j = json.load(f)
-    src_hash = hashlib.sha256(open(KERNELS_SRC, "rb").read()).hexdigest()[:16]
     ent = j.get(kernel_key)
-    if not ent or ent.get("kernels_sha256_16") != src_hash:
+    if not ent or ent.get("kernels_sha256_16") != kernels_source_hash():
         return None
     return ent.get("bytes_per_launch")
 

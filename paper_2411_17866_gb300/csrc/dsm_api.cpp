@@ -514,6 +514,7 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     g.B = h->hp.rsign_B;
     g.n_f = float(h->n);
     g.sign_mode = h->hp.sign_mode;
+    g.mode = h->hp.global_mode;
     g.philox_k0 = static_cast<uint32_t>(h->hp.seed & 0xFFFFFFFFull);
     g.philox_k1 = static_cast<uint32_t>(h->t & 0xFFFFFFFFull);
     cudaStream_t s = S(stream);

@@ -1,0 +1,235 @@
+// The fused round's kernel (DSM_FLAG_FUSED_ROUND): the last local step of a
+// round inside the global step (arXiv 2411.17866, Algorithm 1), in its own
+// translation unit so that it compiles in parallel with the other kernels.
+
+#include "dsm_device.cuh"
+
+namespace dsm {
+namespace {
+
+// K6: the round's last local step fused with the sign-momentum global step.
+// One thread owns 4 elements of every worker: it runs the base optimizer's
+// last step on each worker (writing the worker's optimizer state, but not
+// its new replica, which only feeds the average), then the global step of
+// Algorithm 1 on those elements.  The replicas are not reset: the next
+// round's first local step starts every worker from x.  from_global: the
+// replicas' reset from the previous round is still pending (tau = 1).
+// kVariants: the global step is g.mode (SlowMo, signed SlowMo or Lookahead)
+// instead of Algorithm 1's.
+// A CTA walks its tiles worker by worker; each thread keeps the next
+// kFusedDepth (tile, worker) items in flight with cp.async into its own
+// shared-memory slots (x_i, m_i, v_i, g_i, and x, m with a tile's first worker).
+// Items in flight per thread: 2, or 3 for AdamW with more than 4 workers,
+// whose registers already limit the resident CTAs (measured on GB300: depth 2
+// gives 0.92 / 1.00 of the copy bandwidth on GPT-2 S (AdamW, n = 4) / L
+// (SGD-momentum, n = 8), depth 3 gives 0.85 on GPT-2 M (AdamW, n = 8) where
+// depth 2 gives 0.79).
+constexpr int kFusedStreams = 6;
+__host__ __device__ constexpr int fused_depth(bool adamw, int nw) { return (adamw && nw > 4) ? 3 : 2; }
+__host__ __device__ constexpr size_t fused_smem(int depth) { return size_t(depth) * kFusedStreams * kThreads * sizeof(float4); }
+
+template <bool kAdamW, bool kBf16, int NW, bool kVariants>
+__global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
+                                                                GlobalScalars g, int from_global) {
+    constexpr int kFusedDepth = fused_depth(kAdamW, NW);
+    extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
+    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+    auto slot = [&](int it, int stream) -> float4* {
+        return fsm + (size_t(it % kFusedDepth) * kFusedStreams + stream) * kThreads + threadIdx.x;
+    };
+    // Issue item `it` (tile number it / NW of this CTA, worker it % NW); always commits one group.
+    auto issue = [&](uint32_t it) {
+        const uint32_t q = it / NW, w = it - q * NW;
+        const uint64_t ti = blockIdx.x + uint64_t(q) * gridDim.x;
+        if (ti < p.num_tiles) {
+            const TileDesc t = p.tiles[ti];
+            if (vector_ok(t, e0)) {
+                const uint64_t gi = t.start + e0;
+                const uint64_t o = w * p.d_stride + gi;
+                if (!from_global) cp_async16(slot(it, 0), p.X + o);
+                cp_async16(slot(it, 1), p.opt_m + o);
+                if (kAdamW) cp_async16(slot(it, 2), p.opt_v + o);
+                if (kBf16) cp_async8(slot(it, 3), reinterpret_cast<const __nv_bfloat16*>(p.grad) + o);
+                else cp_async16(slot(it, 3), reinterpret_cast<const float*>(p.grad) + o);
+                if (w == 0) {
+                    cp_async16(slot(it, 4), p.x + gi);
+                    cp_async16(slot(it, 5), p.m + gi);
+                }
+            }
+        }
+        cp_async_commit();
+    };
+    auto take = [&](int it, int stream, float (&v)[4]) {
+        const float4 t = *slot(it, stream);
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+    };
+    uint32_t next_issue = 0;
+    for (int k = 0; k < kFusedDepth; ++k) issue(next_issue++);
+    ThreadStats st;
+    uint32_t it = 0;
+    for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
+        const TileDesc td = p.tiles[ti];
+        const TensorDesc& T = p.tensors[td.tensor];
+        const float lam_l = kAdamW ? T.lam_local : 0.f, lam_g = T.lam_global;
+        const uint64_t gi = td.start + e0;
+        if (vector_ok(td, e0)) {
+            float x[4], m[4], dif[NW][4];
+#pragma unroll
+            for (int w = 0; w < NW; ++w, ++it) {
+                cp_async_wait<kFusedDepth - 1>();  // item `it` has landed
+                float xi[4], mi[4], vi[4], gr[4];
+                if (w == 0) {
+                    take(it, 4, x);
+                    take(it, 5, m);
+                }
+                if (from_global) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) xi[j] = x[j];
+                } else {
+                    take(it, 0, xi);
+                }
+                take(it, 1, mi);
+                if (kAdamW) take(it, 2, vi);
+                if (kBf16) {
+                    const uint2 raw = *reinterpret_cast<const uint2*>(slot(it, 3));
+                    gr[0] = __uint_as_float(raw.x << 16);
+                    gr[1] = __uint_as_float(raw.x & 0xFFFF0000u);
+                    gr[2] = __uint_as_float(raw.y << 16);
+                    gr[3] = __uint_as_float(raw.y & 0xFFFF0000u);
+                } else {
+                    take(it, 3, gr);
+                }
+                const uint64_t o = w * p.d_stride + gi;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (kAdamW) adamw_elem(xi[j], mi[j], vi[j], gr[j], a, lam_l);
+                    else sgdm_elem(xi[j], mi[j], gr[j], sa);
+                    dif[w][j] = __fsub_rn(x[j], xi[j]);
+                }
+                store4(p.opt_m + o, mi);
+                if (kAdamW) store4(p.opt_v + o, vi);
+                // refill the slot just read; the arithmetic above consumed its values, so the
+                // shared-memory reads are complete before the asynchronous copy can overwrite them
+                issue(next_issue++);
+            }
+            float ru[4] = {0.f, 0.f, 0.f, 0.f};
+            if (g.sign_mode != 0) {
+                const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                float d[NW];
+#pragma unroll
+                for (int w = 0; w < NW; ++w) d[w] = dif[w][j];
+                if (kVariants) {
+                    global_elem_rt<NW>(x[j], m[j], d, g, lam_g, ru[j], st);
+                } else {
+                    float unused = 0.f;
+                    global_elem<NW, 0>(x[j], m[j], unused, d, NW, g, lam_g, ru[j], st);
+                }
+            }
+            store4(p.x + gi, x);
+            store4(p.m + gi, m);
+        } else {
+            // this thread issued no copies for the tile; keep the group count in step
+#pragma unroll
+            for (int w = 0; w < NW; ++w, ++it) issue(next_issue++);
+            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
+            for (uint32_t e = e0; e < e1; ++e) {
+                const uint64_t gj = td.start + e;
+                float x = p.x[gj], m = p.m[gj], d[NW];
+#pragma unroll
+                for (int w = 0; w < NW; ++w) {
+                    const uint64_t o = w * p.d_stride + gj;
+                    float xi = from_global ? x : p.X[o], mi = p.opt_m[o];
+                    if (kAdamW) {
+                        float vi = p.opt_v[o];
+                        adamw_elem(xi, mi, vi, load_grad1(p.grad, kBf16, o), a, lam_l);
+                        p.opt_v[o] = vi;
+                    } else {
+                        sgdm_elem(xi, mi, load_grad1(p.grad, kBf16, o), sa);
+                    }
+                    p.opt_m[o] = mi;
+                    d[w] = __fsub_rn(x, xi);
+                }
+                float r = 0.f;
+                if (g.sign_mode != 0) r = philox_unit(word_of(philox_block(gj >> 2, g.philox_k0, g.philox_k1), gj & 3));
+                if (kVariants) {
+                    global_elem_rt<NW>(x, m, d, g, lam_g, r, st);
+                } else {
+                    float unused = 0.f;
+                    global_elem<NW, 0>(x, m, unused, d, NW, g, lam_g, r, st);
+                }
+                p.x[gj] = x;
+                p.m[gj] = m;
+            }
+        }
+        const uint32_t next = ti + gridDim.x;
+        if (next >= p.num_tiles || p.tiles[next].tensor != td.tensor) {  // uniform across the CTA
+            reduce_stats(st, p.partials + ti);
+            st = ThreadStats();
+        } else {
+            zero_partial(p.partials + ti);
+        }
+    }
+    cp_async_wait<0>();  // the groups issued past the last tile are empty; nothing is left in flight
+}
+
+using FusedKernel = void (*)(Problem, AdamScalars, SgdmScalars, GlobalScalars, int);
+
+template <bool kAdamW, bool kBf16, bool kVariants>
+FusedKernel fused_kernel_n(uint32_t n) {
+    switch (n) {
+        case 1: return k_fused_last_global<kAdamW, kBf16, 1, kVariants>;
+        case 2: return k_fused_last_global<kAdamW, kBf16, 2, kVariants>;
+        case 3: return k_fused_last_global<kAdamW, kBf16, 3, kVariants>;
+        case 4: return k_fused_last_global<kAdamW, kBf16, 4, kVariants>;
+        case 5: return k_fused_last_global<kAdamW, kBf16, 5, kVariants>;
+        case 6: return k_fused_last_global<kAdamW, kBf16, 6, kVariants>;
+        case 7: return k_fused_last_global<kAdamW, kBf16, 7, kVariants>;
+        case 8: return k_fused_last_global<kAdamW, kBf16, 8, kVariants>;
+        default: return nullptr;
+    }
+}
+
+template <bool kVariants>
+FusedKernel fused_kernel_v(const Problem& p, bool adamw) {
+    if (adamw) return p.grad_bf16 ? fused_kernel_n<true, true, kVariants>(p.n) : fused_kernel_n<true, false, kVariants>(p.n);
+    return p.grad_bf16 ? fused_kernel_n<false, true, kVariants>(p.n) : fused_kernel_n<false, false, kVariants>(p.n);
+}
+
+FusedKernel fused_kernel_for(const Problem& p, bool adamw) {
+    return p.global_mode == 0 ? fused_kernel_v<false>(p, adamw) : fused_kernel_v<true>(p, adamw);
+}
+
+size_t fused_smem_for(const Problem& p, bool adamw) { return fused_smem(fused_depth(adamw, int(p.n))); }
+
+}  // namespace
+
+bool fused_round_available(const Problem& p) {
+    // the global AdamW step keeps a third stream (v) and runs unfused
+    return p.global_mode >= 0 && p.global_mode <= 3 && p.n >= 1 && p.n <= kMaxUnrolledWorkers;
+}
+
+cudaError_t query_fused_shape(const Problem& p, LaunchShape* out) {
+    if (!fused_round_available(p)) return cudaSuccess;
+    const FusedKernel fk = fused_kernel_for(p, p.opt_v != nullptr);
+    const size_t smem = fused_smem_for(p, p.opt_v != nullptr);
+    cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    out->grid_fused = grid_for(fk, out->sms, smem);
+    return cudaSuccess;
+}
+
+cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
+                                     const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s) {
+    if (!fused_round_available(p)) return cudaErrorInvalidValue;
+    const int grid = clamp_grid(ls.grid_fused, p.num_tiles);
+    if (grid == 0) return cudaSuccess;
+    fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, fused_smem_for(p, p.opt_v != nullptr), s>>>(
+        p, a, sa, g, from_x ? 1 : 0);
+    return cudaGetLastError();
+}
+
+}  // namespace dsm

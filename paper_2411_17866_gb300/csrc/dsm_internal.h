@@ -102,6 +102,7 @@ struct GlobalScalars {
     float B;               // randomized-sign bound
     float n_f;             // n as float (divisor of the average)
     int sign_mode;
+    int mode;              // DSM_GLOBAL_*: read by the fused round's kernel for the ablation variants
     uint32_t philox_k0, philox_k1;
 };
 
@@ -130,6 +131,7 @@ cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const Sgd
                               cudaStream_t s);
 // The fused round's last local step + sign-momentum global step (n <= 8).
 bool fused_round_available(const Problem& p);
+cudaError_t query_fused_shape(const Problem& p, LaunchShape* out);  // sets grid_fused (out->sms must be set)
 cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
                                      const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s);
 cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);

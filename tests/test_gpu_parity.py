@@ -93,11 +93,14 @@ VARIANTS = [
 ]
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
 @pytest.mark.parametrize("layout_name", ["ragged", "mini"])
 @pytest.mark.parametrize("name,hp,n,tau", VARIANTS, ids=[c[0] for c in VARIANTS])
-def test_global_variants_bitexact(layout_name, name, hp, n, tau):
-    """The ablations' global steps (SlowMo, signed SlowMo, Lookahead, global AdamW), three rounds."""
+def test_global_variants_bitexact(layout_name, name, hp, n, tau, fused):
+    """The ablations' global steps (SlowMo, signed SlowMo, Lookahead, global AdamW), three rounds,
+    in the unfused and the fused round (global AdamW and n > 8 fall back to unfused)."""
     tensors = RAGGED if layout_name == "ragged" else MINI
+    hp = dataclasses.replace(hp, flags=W.FLAG_FUSED_ROUND if fused else 0)
     run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
     ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
     for _ in range(3):
