@@ -32,7 +32,10 @@
  * Errors
  *   Every int-returning call returns DSM_OK (0) or a negative DSM_E* code
  *   and never aborts the process; dsm_last_error() gives a message for the
- *   calling thread's last failure.
+ *   calling thread's last failure.  A call that fails argument or order
+ *   checks (DSM_EINVAL, DSM_ERANGE, DSM_ESTATE, ...) changes nothing.  After
+ *   DSM_ECUDA from a call that enqueues work, the device state is whatever
+ *   the failed CUDA call left: restore a checkpoint or create a new handle.
  *
  * Thread safety: a handle is not thread-safe; distinct handles are
  * independent.

@@ -238,23 +238,24 @@ cudaMemcpyKind copy_kind(int other_is_device, bool to_device) {
     return to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost;
 }
 
-// Scalars of the next local step (count j + 1); advances the beta powers.
-void next_local_scalars(dsm_handle* h, AdamScalars* a, SgdmScalars* sa) {
+// Scalars of the next local step (count j + 1) and the beta powers that step
+// reaches; the handle is updated only once the step is launched or deferred.
+void next_local_scalars(const dsm_handle* h, AdamScalars* a, SgdmScalars* sa, double* nb1, double* nb2) {
     *a = AdamScalars{};
     *sa = SgdmScalars{};
+    *nb1 = h->b1_pow;
+    *nb2 = h->b2_pow;
     if (h->hp.base == DSM_BASE_ADAMW) {
-        const double nb1 = h->b1_pow * double(h->hp.b1);
-        const double nb2 = h->b2_pow * double(h->hp.b2);
+        *nb1 = h->b1_pow * double(h->hp.b1);
+        *nb2 = h->b2_pow * double(h->hp.b2);
         a->b1 = h->hp.b1;
         a->omb1 = float(1.0 - double(h->hp.b1));
         a->b2 = h->hp.b2;
         a->omb2 = float(1.0 - double(h->hp.b2));
-        a->bc1 = float(1.0 - nb1);
-        a->bc2 = float(1.0 - nb2);
+        a->bc1 = float(1.0 - *nb1);
+        a->bc2 = float(1.0 - *nb2);
         a->lr = h->gamma;
         a->eps = h->hp.eps;
-        h->b1_pow = nb1;
-        h->b2_pow = nb2;
     } else {
         sa->mu = h->hp.mu;
         sa->lr = h->gamma;
@@ -473,15 +474,18 @@ int dsm_local_step(dsm_handle* h, dsm_stream_t stream) {
     // step count j = t*tau + k + 1; beta^j by successive float64 products
     AdamScalars a;
     SgdmScalars sa;
-    next_local_scalars(h, &a, &sa);
+    double nb1, nb2;
+    next_local_scalars(h, &a, &sa, &nb1, &nb2);
     if (h->fused && h->k + 1 == h->tau) {  // the last step runs inside dsm_global_step
         h->pending_a = a;
         h->pending_sa = sa;
         h->last_pending = true;
     } else {
         cudaError_t err = launch_local(h, a, sa, S(stream));
-        if (err != cudaSuccess) return cuda_fail(err, "launch local step");
+        if (err != cudaSuccess) return cuda_fail(err, "launch local step");  // the handle is unchanged
     }
+    h->b1_pow = nb1;
+    h->b2_pow = nb2;
     h->j += 1;
     h->k += 1;
     return DSM_OK;
