@@ -202,7 +202,25 @@ class ClockSampler:
 
     def __init__(self, gpu_index):
         self.proc = None
-        self.gpu = gpu_index
+        self.gpu = self.smi_id(gpu_index)
+
+    @staticmethod
+    def smi_id(local_index: int) -> str:
+        """nvidia-smi's -i for CUDA device `local_index`: nvidia-smi ignores CUDA_VISIBLE_DEVICES, so use the
+        device's UUID (or the listed id) rather than the CUDA index."""
+        try:
+            import torch
+            uuid = str(torch.cuda.get_device_properties(local_index).uuid)
+            if uuid:
+                return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+        except Exception:
+            pass
+        visible = os.environ.get("CUDA_VISIBLE_DEVICES", "").strip()
+        if visible:
+            ids = [v.strip() for v in visible.split(",") if v.strip()]
+            if local_index < len(ids):
+                return ids[local_index]
+        return str(local_index)
 
     def start(self):
         try:
@@ -244,7 +262,7 @@ class ClockSampler:
                 if r[key].lower() == "active":
                     reasons.add(name)
         return {"sm_mhz": statistics.median(r["sm"] for r in loaded), "sm_max_mhz": rows[0]["max"],
-                "reasons": sorted(reasons), "samples": len(rows), "power_w_max": pmax}
+                "reasons": sorted(reasons), "samples": len(rows), "power_w_max": pmax, "gpu": self.gpu}
 
 
 def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, rounds=1):
