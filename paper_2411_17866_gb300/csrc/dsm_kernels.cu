@@ -494,14 +494,20 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     out->sms = sms;
     out->grid_init = grid_for(k_init, sms);
     out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms) : grid_for(k_grad_fill<false>, sms);
-    out->grid_adamw = p.grad_bf16 ? grid_for(k_local_adamw<true, false>, sms) : grid_for(k_local_adamw<false, false>, sms);
+    // The AdamW step fits 4 CTAs per SM.  With fp32 gradients it streams better with 3 (GB300, GPT-2 S,
+    // n = 4: 1.00 of the copy bandwidth with 3, 0.95 with 4); with bf16 gradients 4 are better
+    // (GPT-2 M, n = 8: 0.97 with 4, 0.90 with 3; GPT-2 XL, n = 4: 0.96 with 4, 0.87 with 3).
+    const int kAdamwCtasPerSm = p.grad_bf16 ? 4 : 3;
+    out->grid_adamw = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, false>, sms)
+                                           : grid_for(k_local_adamw<false, false>, sms), kAdamwCtasPerSm * sms);
     // The SGD-momentum step fits 6 CTAs per SM, but 4 stream better (GB300, GPT-2 L layout, n = 8:
     // 0.96 of the copy bandwidth with 4, 0.91 with 6, 0.91 with 3), as many as the AdamW step holds.
     constexpr int kSgdmCtasPerSm = 4;
     out->grid_sgdm = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, false>, sms)
                                           : grid_for(k_local_sgdm<false, false>, sms), kSgdmCtasPerSm * sms);
     if (fused_round_available(p)) {
-        out->grid_adamw_from_x = p.grad_bf16 ? grid_for(k_local_adamw<true, true>, sms) : grid_for(k_local_adamw<false, true>, sms);
+        out->grid_adamw_from_x = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, true>, sms)
+                                                      : grid_for(k_local_adamw<false, true>, sms), kAdamwCtasPerSm * sms);
         out->grid_sgdm_from_x = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, true>, sms)
                                                      : grid_for(k_local_sgdm<false, true>, sms), kSgdmCtasPerSm * sms);
         cudaError_t e = query_fused_shape(p, out);
