@@ -133,6 +133,19 @@ __device__ __forceinline__ float grad_value(float a, float s2, float u2) {
     return __fadd_rn(a, __fmul_rn(s2, __fsub_rn(u2, 0.5f)));
 }
 
+// The same products with one multiplication per draw.  u - 1/2 equals
+// (h24 - 2^23) * 2^-24 exactly, and for |s| >= 2^-102 so is s * 2^-24
+// (a normal number), so s*(u - 1/2) and (s*2^-24)*(h24 - 2^23) are the same
+// real number and round to the same float.  `sp` is s*2^-24; the draw
+// enters as the signed integer h24 - 2^23, which converts exactly.
+constexpr float kMinPrescaled = 1.9721522630525295e-31f;  // 2^-102
+__device__ __forceinline__ float centred_even(uint64_t h) {
+    return __int2float_rn(static_cast<int32_t>(static_cast<uint32_t>(h >> 40)) - 0x800000);
+}
+__device__ __forceinline__ float centred_odd(uint64_t h) {
+    return __int2float_rn(static_cast<int32_t>(static_cast<uint32_t>(h >> 16) & 0xFFFFFFu) - 0x800000);
+}
+
 // AdamW (Appendix A): m <- b1 m + (1-b1) g; v <- b2 v + (1-b2) g*g;
 // x <- x - lr (mhat/(sqrt(vhat)+eps) + lam x), mhat = m/bc1, vhat = v/bc2.
 __device__ __forceinline__ void adamw_elem(float& x, float& m, float& v, float g, const AdamScalars& a, float lam) {

@@ -58,6 +58,38 @@ __global__ void __launch_bounds__(kThreads) k_init(Problem p, uint64_t key_init,
 // K1: synthetic gradients of one local step for every worker.  Bound by the
 // integer work of the hash (one 64-bit SplitMix64 output per two elements
 // and per draw family), not by its write stream.
+template <bool kBf16, bool kPrescaled>
+__device__ __forceinline__ void grad_fill4(const Problem& p, const GradKeys& k, uint64_t gi, float s, float s2) {
+    // even gi: elements gi..gi+3 use outputs gi/2+1, gi/2+2; output j of any
+    // family is finalise(key + j*gamma), and j*gamma is shared by all families
+    const uint64_t jg0 = ((gi >> 1) + 1) * kGoldenGamma, jg1 = jg0 + kGoldenGamma;
+    const uint64_t h0 = sm64_finalise(k.step + jg0), h1 = sm64_finalise(k.step + jg1);
+    float a[4];
+    if (kPrescaled) {
+        a[0] = __fmul_rn(s, centred_even(h0)); a[1] = __fmul_rn(s, centred_odd(h0));
+        a[2] = __fmul_rn(s, centred_even(h1)); a[3] = __fmul_rn(s, centred_odd(h1));
+    } else {
+        a[0] = step_term(s, draw_even(h0)); a[1] = step_term(s, draw_odd(h0));
+        a[2] = step_term(s, draw_even(h1)); a[3] = step_term(s, draw_odd(h1));
+    }
+    for (uint32_t w = 0; w < p.n; ++w) {
+        const uint64_t q0 = sm64_finalise(k.worker[w] + jg0), q1 = sm64_finalise(k.worker[w] + jg1);
+        float g[4];
+        if (kPrescaled) {
+            g[0] = __fadd_rn(a[0], __fmul_rn(s2, centred_even(q0)));
+            g[1] = __fadd_rn(a[1], __fmul_rn(s2, centred_odd(q0)));
+            g[2] = __fadd_rn(a[2], __fmul_rn(s2, centred_even(q1)));
+            g[3] = __fadd_rn(a[3], __fmul_rn(s2, centred_odd(q1)));
+        } else {
+            g[0] = grad_value(a[0], s2, draw_even(q0)); g[1] = grad_value(a[1], s2, draw_odd(q0));
+            g[2] = grad_value(a[2], s2, draw_even(q1)); g[3] = grad_value(a[3], s2, draw_odd(q1));
+        }
+        const uint64_t o = w * p.d_stride + gi;
+        if (kBf16) store4_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
+        else store4(reinterpret_cast<float*>(p.grad) + o, g);
+    }
+}
+
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
@@ -66,20 +98,10 @@ __global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
         const TensorDesc& T = p.tensors[td.tensor];
         const float s = T.scale, s2 = T.scale2;
         if (vector_ok(td, e0)) {
-            const uint64_t gi = td.start + e0;  // even: elements gi..gi+3 use outputs gi/2+1, gi/2+2
-            // output j of any family is finalise(key + j*gamma): j*gamma is shared by all families
-            const uint64_t jg0 = ((gi >> 1) + 1) * kGoldenGamma, jg1 = jg0 + kGoldenGamma;
-            const uint64_t h0 = sm64_finalise(k.step + jg0), h1 = sm64_finalise(k.step + jg1);
-            const float a[4] = {step_term(s, draw_even(h0)), step_term(s, draw_odd(h0)),
-                                step_term(s, draw_even(h1)), step_term(s, draw_odd(h1))};
-            for (uint32_t w = 0; w < p.n; ++w) {
-                const uint64_t q0 = sm64_finalise(k.worker[w] + jg0), q1 = sm64_finalise(k.worker[w] + jg1);
-                const float g[4] = {grad_value(a[0], s2, draw_even(q0)), grad_value(a[1], s2, draw_odd(q0)),
-                                    grad_value(a[2], s2, draw_even(q1)), grad_value(a[3], s2, draw_odd(q1))};
-                const uint64_t o = w * p.d_stride + gi;
-                if (kBf16) store4_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
-                else store4(reinterpret_cast<float*>(p.grad) + o, g);
-            }
+            if (fabsf(s) >= kMinPrescaled && fabsf(s2) >= kMinPrescaled)
+                grad_fill4<kBf16, true>(p, k, td.start + e0, __fmul_rn(s, kTwoPowM24), __fmul_rn(s2, kTwoPowM24));
+            else
+                grad_fill4<kBf16, false>(p, k, td.start + e0, s, s2);
         } else {
             const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
             for (uint32_t e = e0; e < e1; ++e) {

@@ -381,6 +381,26 @@ def test_zero_gradients():
     run.close()
 
 
+@pytest.mark.parametrize("grad_dtype", [W.F32, W.BF16], ids=["f32", "bf16"])
+def test_gradient_scales_across_the_prescaled_limit(grad_dtype):
+    """K1 multiplies by s*2^-24 when both s and 0.1*s are at least 2^-102 and by s otherwise; both forms
+    must give the oracle's bits.  Scales on either side of the limit, a huge one and zero, every worker."""
+    scales = [2.0 ** -102, 2.0 ** -98, 1e-35, 1e-30, 3e37, 0.0, 1e-3]
+    tensors = tuple(W.Tensor(f"s{i}", numel, W.KIND_WEIGHT, sc)
+                    for i, (sc, numel) in enumerate(zip(scales, [4096, 1031, 2048, 4100, 1024, 64, 3000])))
+    n = 3
+    hp = dataclasses.replace(ADAMW, grad_dtype=grad_dtype, seed=9)
+    run = dsm.DistributedSignMomentum(tensors, n, 1, hp)
+    ora = O.OracleRun(tensors, n, 1, hp)
+    for step in (0, 5):
+        run.fill_synthetic_grads(step)
+        for w in range(n):
+            g = run.read(dsm.BUF_GRAD, w).to(torch.float32).numpy()
+            want = O.synthetic_grad(ora.elems, ora.scale, hp.seed, step, w, grad_dtype)
+            assert_bitexact(g, want, f"grad step {step} worker {w}")
+    run.close()
+
+
 def test_guard_regions_detect_an_overrun():
     """A byte written past the end of the tensor table (a planted host-side write) is reported."""
     run = dsm.DistributedSignMomentum(MINI, 2, 1, ADAMW)
