@@ -334,6 +334,8 @@ GLOBAL_SIGNED_SLOWMO = 2   # Sec. 5, signed SlowMo
 GLOBAL_LOOKAHEAD = 3       # Sec. 5, Lookahead (Eq. (model-update) replaced)
 GLOBAL_ADAMW = 4           # Appendix, Algorithm "global AdamW"
 
+FLAG_RESET_LOCAL_STATE = 2  # hp.flags bit: restart each worker's optimizer every round
+
 
 def worker_average(x, X, dt):
     """Delta = (1/n) sum_i (x - x_i), summed over i = 0..n-1 in order (the all-reduce average)."""
@@ -460,7 +462,10 @@ class OracleRun:
 
     Worker optimizer states persist across rounds and are never averaged;
     only the model is synchronised (Algorithm 1, last step).  AdamW's step
-    count is j = t*tau + k + 1.
+    count is j = t*tau + k + 1.  Algorithm 1 leaves the base optimizer's
+    state at a synchronisation open; with hp.flags & FLAG_RESET_LOCAL_STATE
+    every round instead restarts each worker's optimizer from scratch: its
+    state is zero at the start of the round and j = k + 1.
     """
 
     def __init__(self, tensors, n, tau, hp, elems=None, x0=None, dtype=np.float32,
@@ -490,6 +495,7 @@ class OracleRun:
         self.opt_v = [np.zeros_like(self.x) for _ in range(self.n)] if hp.base == 0 else None
         self.global_mode = getattr(hp, "global_mode", GLOBAL_SIGN_MOMENTUM)
         self.gv = np.zeros_like(self.x) if self.global_mode == GLOBAL_ADAMW else None
+        self.reset_local = bool(getattr(hp, "flags", 0) & FLAG_RESET_LOCAL_STATE)
         self.t = 0
         self.k = 0
         self.gamma = hp.lr
@@ -504,12 +510,13 @@ class OracleRun:
         """Local step k of the current round for every worker, Eq. (local-steps)."""
         assert self.k < self.tau
         step = self.t * self.tau + self.k
+        j = self.k + 1 if self.reset_local else step + 1
         hp = self.hp
         for i in range(self.n):
             g = self.grads(step, i) if grads is None else np.asarray(grads[i], dtype=np.float32)
             if hp.base == 0:
                 self.X[i], self.opt_m[i], self.opt_v[i] = adamw_step(
-                    self.X[i], self.opt_m[i], self.opt_v[i], g, step + 1,
+                    self.X[i], self.opt_m[i], self.opt_v[i], g, j,
                     self.gamma, hp.b1, hp.b2, hp.eps, self.wd_local, self.dt)
             else:
                 self.X[i], self.opt_m[i] = sgdm_step(self.X[i], self.opt_m[i], g, self.gamma, hp.mu, self.dt)
@@ -547,6 +554,10 @@ class OracleRun:
         self.last_inter = inter
         self.x, self.m = x_new, m_new
         self.X = [x_new.copy() for _ in range(self.n)]
+        if self.reset_local:
+            self.opt_m = [np.zeros_like(self.x) for _ in range(self.n)]
+            if self.opt_v is not None:
+                self.opt_v = [np.zeros_like(self.x) for _ in range(self.n)]
         self.t += 1
         self.k = 0
 

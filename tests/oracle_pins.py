@@ -533,6 +533,48 @@ def pin_global_adamw_vs_torch(o):
         assert np.allclose(run.x, p.detach().numpy(), rtol=1e-10, atol=1e-12)
 
 
+def pin_local_state_across_rounds(o):
+    """Algorithm 1 synchronises only the model.  By default a worker's AdamW keeps its moments and its
+    step count across rounds: one torch.optim.AdamW per worker for the whole run.  With
+    FLAG_RESET_LOCAL_STATE every round starts a new torch.optim.AdamW per worker.  Between rounds the
+    oracle's global step (itself pinned by the worked example) averages and synchronises."""
+    import torch
+    rng = np.random.default_rng(21)
+    d, n, tau, rounds = 512, 3, 3, 3
+    finals = []
+    for flags in (0, W.FLAG_RESET_LOCAL_STATE):
+        hp = W.HParams(flags=flags)
+        x0 = rng.standard_normal(d).astype(np.float32)
+        run = o.OracleRun(W.flat_layout(d, 1e-3), n, tau, hp, x0=x0, dtype=np.float64)
+        x, m = x0.astype(np.float64), np.zeros(d)
+        params = [torch.tensor(x.copy(), dtype=torch.float64, requires_grad=True) for _ in range(n)]
+
+        def new_opt(p):
+            return torch.optim.AdamW([p], lr=o.f32(hp.lr), betas=(o.f32(hp.b1), o.f32(hp.b2)),
+                                     eps=o.f32(hp.eps), weight_decay=o.f32(hp.wd), foreach=False)
+
+        opts = [new_opt(p) for p in params]
+        for t in range(rounds):
+            grads = [[(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(n)] for _ in range(tau)]
+            if flags and t:
+                opts = [new_opt(p) for p in params]
+            for k in range(tau):
+                for i in range(n):
+                    params[i].grad = torch.tensor(grads[k][i].astype(np.float64))
+                    opts[i].step()
+            X = [p.detach().numpy().copy() for p in params]
+            x, m, _ = o.global_step(x, m, X, hp.lr, hp.g_b1, hp.g_b2, hp.g_eta, np.full(d, o.f32(hp.g_wd)),
+                                    0, hp.rsign_B, None, np.dtype(np.float64))
+            with torch.no_grad():
+                for p in params:
+                    p.copy_(torch.from_numpy(x))
+            run.run_round(grads)
+            assert np.max(np.abs(run.x - x)) <= 1e-12 * (1 + np.max(np.abs(x))), (flags, t)
+            assert np.max(np.abs(run.m - m)) <= 1e-9 * (1e-6 + np.max(np.abs(m))), (flags, t)
+        finals.append(run.opt_m[0].copy())
+    assert np.all(finals[1] == 0.0) and np.any(finals[0] != 0.0)
+
+
 def pin_cosine_schedule(o):
     """Closed-form points of warm-up + cosine decay: P/W at step 0, P at the end of the warm-up,
     (P + F)/2 halfway through the decay, F at and after the last step; monotone decay."""
@@ -554,4 +596,4 @@ PINS = [pin_worked_example, pin_splitmix64, pin_philox, pin_philox_uniform_mappi
         pin_lion, pin_signsgd_momentum, pin_identical_workers, pin_tau1_pseudo_gradient,
         pin_sign_range, pin_lemma1, pin_stats, pin_subset_mode, pin_fp32_vs_fp64,
         pin_slowmo_heavy_ball, pin_lookahead_slow_weights, pin_signed_slowmo_signsgd, pin_global_adamw_vs_torch,
-        pin_cosine_schedule]
+        pin_cosine_schedule, pin_local_state_across_rounds]

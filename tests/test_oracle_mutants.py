@@ -88,6 +88,10 @@ MUTANTS = [
      [P.pin_global_adamw_vs_torch]),
     ("global_adamw_no_inv_gamma", "g = T(1.0 / f32(gamma)) * delta", "g = delta",
      [P.pin_global_adamw_vs_torch]),
+    ("reset_keeps_step_count", "j = self.k + 1 if self.reset_local else step + 1", "j = step + 1",
+     [P.pin_local_state_across_rounds]),
+    ("reset_keeps_moments", "            self.opt_m = [np.zeros_like(self.x) for _ in range(self.n)]\n",
+     "            pass\n", [P.pin_local_state_across_rounds]),
     ("subset_tensor_lookup", "self.tensor_of = np.searchsorted(self.starts, self.elems, side=\"right\") - 1",
      "self.tensor_of = np.searchsorted(self.starts, self.elems, side=\"left\") - 1",
      [P.pin_subset_mode, P.pin_stats]),

@@ -41,8 +41,11 @@ GLOBAL_SLOWMO = 1
 GLOBAL_SIGNED_SLOWMO = 2
 GLOBAL_LOOKAHEAD = 3
 GLOBAL_ADAMW = 4
-# Execution flags
+# Flags: FUSED_ROUND is an execution option (the results do not depend on it);
+# RESET_LOCAL_STATE selects a variant of the method (every round starts each
+# worker's base-optimizer state from zero and restarts AdamW's step count).
 FLAG_FUSED_ROUND = 1
+FLAG_RESET_LOCAL_STATE = 2
 
 VOCAB = 50257
 CONTEXT = 1024
@@ -76,7 +79,7 @@ class HParams:
     seed: int = 0
     global_mode: int = 0      # GLOBAL_* below
     g_eps: float = 1e-8       # epsilon of the global AdamW step
-    flags: int = 0            # FLAG_* below (execution options; the results do not depend on them)
+    flags: int = 0            # FLAG_* above
 
 
 @dataclasses.dataclass(frozen=True)
