@@ -110,6 +110,18 @@ extern "C" {
  * dsm_local_step and dsm_global_step. */
 #define DSM_FLAG_FUSED_ROUND 1u
 
+/* Restart the base optimizer every round.  Algorithm 1 synchronises only
+ * the model (its last step) and leaves open what becomes of each worker's
+ * base-optimizer state; by default that state (AdamW moments, SGD-momentum
+ * buffer) persists across rounds and AdamW counts j = t*tau + k + 1.  With
+ * this flag every round instead starts each worker's base optimizer afresh,
+ * as if a new optimizer were built at each synchronisation: its state is
+ * zero at the round's first local step and AdamW counts j = k + 1.  Reading
+ * DSM_BUF_OPT_M / DSM_BUF_OPT_V between rounds returns zeros.  The zeroing
+ * is lazy: the round's first local step reads no state, and the fused
+ * round's last local step writes none (the next round would discard it). */
+#define DSM_FLAG_RESET_LOCAL_STATE 2u
+
 /* Buffers for dsm_read_params / dsm_write_params. */
 #define DSM_BUF_X        0  /* global model x_{t,0} (fp32, d) */
 #define DSM_BUF_M        1  /* global momentum m_t (fp32, d) */
@@ -243,8 +255,8 @@ int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream
  * the base optimizer's update of each replica from its gradient buffer.
  * AdamW's bias corrections use step count j = t*tau + k + 1 (the
  * base-optimizer states persist across rounds; only the model is
- * synchronised).  DSM_ESTATE if tau local steps were already done in this
- * round.  Asynchronous. */
+ * synchronised), or j = k + 1 with DSM_FLAG_RESET_LOCAL_STATE.  DSM_ESTATE
+ * if tau local steps were already done in this round.  Asynchronous. */
 int dsm_local_step(dsm_handle* h, dsm_stream_t stream);
 
 /* Global step of Algorithm 1 after the round's tau local steps (else
@@ -292,8 +304,9 @@ int dsm_cosine_gamma(float peak, float final_ratio, uint64_t warmup_steps, uint6
                      float* gamma);
 
 /* Set the round counter t of Algorithm 1 (checkpoint restore): it keys the
- * randomized sign and fixes the AdamW step counts j = t*tau + k + 1 and the
- * global AdamW count t + 1.  Only between rounds, else DSM_ESTATE. */
+ * randomized sign and fixes the AdamW step counts j = t*tau + k + 1 (j = k + 1
+ * with DSM_FLAG_RESET_LOCAL_STATE) and the global AdamW count t + 1.  Only
+ * between rounds, else DSM_ESTATE. */
 int dsm_set_round(dsm_handle* h, uint64_t round);
 
 /* Describe the handle (sizes, t and k of Algorithm 1, gamma_t) into *out.

@@ -105,7 +105,8 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
         return fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
     if (hp->grad_dtype != DSM_F32 && hp->grad_dtype != DSM_BF16)
         return fail(DSM_EINVAL, "gradient dtype %d unknown", hp->grad_dtype);
-    if (hp->flags & ~DSM_FLAG_FUSED_ROUND) return fail(DSM_EINVAL, "unknown bits in hparams.flags");
+    if (hp->flags & ~(DSM_FLAG_FUSED_ROUND | DSM_FLAG_RESET_LOCAL_STATE))
+        return fail(DSM_EINVAL, "unknown bits in hparams.flags");
 
     uint64_t d = 0, tiles = 0;
     for (uint32_t i = 0; i < layout->count; ++i) {
@@ -190,9 +191,12 @@ struct dsm_handle {
     bool fused = false;           // flag set and a fused kernel exists for this problem
     bool replicas_stale = false;  // the replicas' reset to x is pending
     bool last_pending = false;    // the round's last local step waits for the global step
+    // DSM_FLAG_RESET_LOCAL_STATE
+    bool reset_local = false;     // every round restarts the base optimizer
+    bool states_zero = false;     // the base-optimizer states are zero; their zeroing in memory is pending
     AdamScalars pending_a{};
     SgdmScalars pending_sa{};
-    uint64_t j = 0;        // local steps done since the start (AdamW step count)
+    uint64_t j = 0;        // AdamW step count of the last local step (restarts each round with the reset flag)
 };
 
 namespace {
@@ -263,10 +267,10 @@ void next_local_scalars(const dsm_handle* h, AdamScalars* a, SgdmScalars* sa, do
 }
 
 cudaError_t launch_local(dsm_handle* h, const AdamScalars& a, const SgdmScalars& sa, cudaStream_t s) {
-    const bool from_x = h->replicas_stale;
-    cudaError_t err = h->hp.base == DSM_BASE_ADAMW ? launch_local_adamw(h->prob, h->shape, a, from_x, s)
-                                                   : launch_local_sgdm(h->prob, h->shape, sa, from_x, s);
-    if (err == cudaSuccess) h->replicas_stale = false;
+    const bool from_x = h->replicas_stale, zero_state = h->states_zero;
+    cudaError_t err = h->hp.base == DSM_BASE_ADAMW ? launch_local_adamw(h->prob, h->shape, a, from_x, zero_state, s)
+                                                   : launch_local_sgdm(h->prob, h->shape, sa, from_x, zero_state, s);
+    if (err == cudaSuccess) h->replicas_stale = h->states_zero = false;
     return err;
 }
 
@@ -286,6 +290,26 @@ int materialize_replicas(dsm_handle* h, cudaStream_t s) {
     if (err != cudaSuccess) return cuda_fail(err, "reset the replicas");
     h->replicas_stale = false;
     return DSM_OK;
+}
+
+// Zeroes the base-optimizer states in memory (the restart DSM_FLAG_RESET_LOCAL_STATE left pending).
+int materialize_states(dsm_handle* h, cudaStream_t s) {
+    if (!h->states_zero) return DSM_OK;
+    const size_t bytes = size_t(h->n) * h->al.d_stride * 4;
+    cudaError_t err = cudaMemsetAsync(h->prob.opt_m, 0, bytes, s);
+    if (err == cudaSuccess && h->prob.opt_v) err = cudaMemsetAsync(h->prob.opt_v, 0, bytes, s);
+    if (err != cudaSuccess) return cuda_fail(err, "zero the base-optimizer states");
+    h->states_zero = false;
+    return DSM_OK;
+}
+
+// After a global step: the restart of the base optimizer (if the flag asks for it) becomes pending,
+// and AdamW's step count starts again at 1.
+void begin_next_round_states(dsm_handle* h) {
+    if (!h->reset_local) return;
+    h->states_zero = true;
+    h->b1_pow = h->b2_pow = 1.0;
+    h->j = 0;
 }
 
 }  // namespace
@@ -333,6 +357,7 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     h->al = al;
     h->arena = static_cast<char*>(dev_arena);
     h->gamma = hp->lr;
+    h->reset_local = (hp->flags & DSM_FLAG_RESET_LOCAL_STATE) != 0;
 
     // tensor and tile tables
     h->tensors.resize(al.num_tensors);
@@ -524,10 +549,13 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     cudaStream_t s = S(stream);
     cudaError_t err;
     if (h->last_pending) {  // fused round: last local step + global step, reset left pending
-        err = launch_fused_last_global(h->prob, h->shape, h->pending_a, h->pending_sa, g, h->replicas_stale, s);
+        const int opts = (h->replicas_stale ? kFusedFromX : 0) | (h->states_zero ? kFusedZeroState : 0) |
+                         (h->reset_local ? kFusedDropState : 0);
+        err = launch_fused_last_global(h->prob, h->shape, h->pending_a, h->pending_sa, g, opts, s);
         if (err != cudaSuccess) return cuda_fail(err, "launch fused last local step and global step");
         h->last_pending = false;
         h->replicas_stale = true;
+        h->states_zero = false;  // (set again below when the round restarts the base optimizer)
     } else {
         int rc = materialize_replicas(h, s);
         if (rc != DSM_OK) return rc;
@@ -540,6 +568,7 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     h->k = 0;
     h->gb1_pow = ngb1;
     h->gb2_pow = ngb2;
+    begin_next_round_states(h);
     if (stats) {
         err = cudaMemcpyAsync(stats, h->prob.stats, size_t(h->al.num_tensors) * sizeof(TensorStats),
                               cudaMemcpyDeviceToHost, s);
@@ -571,8 +600,19 @@ int dsm_read_params(dsm_handle* h, int which, uint32_t worker, void* dst, uint64
         if (rc != DSM_OK) return rc;
     }
     if (which == DSM_BUF_REPLICA && h->replicas_stale) src = reinterpret_cast<char*>(h->prob.x + offset);
+    cudaError_t err;
+    if ((which == DSM_BUF_OPT_M || which == DSM_BUF_OPT_V) && h->states_zero) {  // restart pending: zeros
+        if (dst_is_device) {
+            err = cudaMemsetAsync(dst, 0, count * es, S(stream));
+            if (err != cudaSuccess) return cuda_fail(err, "read buffer");
+            return DSM_OK;
+        }
+        if ((err = cudaStreamSynchronize(S(stream))) != cudaSuccess) return cuda_fail(err, "synchronise before read");
+        std::memset(dst, 0, count * es);
+        return DSM_OK;
+    }
     const cudaMemcpyKind kind = copy_kind(dst_is_device, false);
-    cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
+    err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "read buffer");
     if (!dst_is_device && (err = cudaStreamSynchronize(S(stream))) != cudaSuccess)
         return cuda_fail(err, "synchronise after read");
@@ -591,6 +631,8 @@ int dsm_write_params(dsm_handle* h, int which, uint32_t worker, const void* src,
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     if ((rc = materialize_pending(h, S(stream))) != DSM_OK) return rc;
     if ((rc = materialize_replicas(h, S(stream))) != DSM_OK) return rc;
+    if ((which == DSM_BUF_OPT_M || which == DSM_BUF_OPT_V) && (rc = materialize_states(h, S(stream))) != DSM_OK)
+        return rc;
     const cudaMemcpyKind kind = copy_kind(src_is_device, true);
     cudaError_t err = cudaMemcpyAsync(dst, src, count * es, kind, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "write buffer");
@@ -624,7 +666,7 @@ int dsm_set_round(dsm_handle* h, uint64_t round) {
     if (!h) return fail(DSM_EINVAL, "handle is NULL");
     if (h->k != 0) return fail(DSM_ESTATE, "the round counter can change only between rounds");
     h->t = round;
-    h->j = round * h->tau;
+    h->j = h->reset_local ? 0 : round * h->tau;
     double p1 = 1.0, p2 = 1.0;
     for (uint64_t i = 0; i < h->j; ++i) {
         p1 *= double(h->hp.b1);

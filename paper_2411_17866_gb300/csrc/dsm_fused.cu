@@ -12,8 +12,11 @@ namespace {
 // last step on each worker (writing the worker's optimizer state, but not
 // its new replica, which only feeds the average), then the global step of
 // Algorithm 1 on those elements.  The replicas are not reset: the next
-// round's first local step starts every worker from x.  from_global: the
-// replicas' reset from the previous round is still pending (tau = 1).
+// round's first local step starts every worker from x.  opts (kFused* bits):
+// kFusedFromX, the replicas' reset from the previous round is still pending
+// (tau = 1); kFusedZeroState, the base-optimizer states are zero and not read
+// (the round restarts the base optimizer and tau = 1); kFusedDropState, the
+// new states are not written (the round restarts the base optimizer).
 // kVariants: the global step is g.mode (SlowMo, signed SlowMo or Lookahead)
 // instead of Algorithm 1's.
 // A CTA walks its tiles worker by worker; each thread keeps the next
@@ -30,8 +33,10 @@ __host__ __device__ constexpr size_t fused_smem(int depth) { return size_t(depth
 
 template <bool kAdamW, bool kBf16, int NW, bool kVariants>
 __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
-                                                                GlobalScalars g, int from_global) {
+                                                                GlobalScalars g, int opts) {
     constexpr int kFusedDepth = fused_depth(kAdamW, NW);
+    const bool from_global = opts & kFusedFromX, zero_state = opts & kFusedZeroState,
+               keep_state = !(opts & kFusedDropState);
     extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     auto slot = [&](int it, int stream) -> float4* {
@@ -47,8 +52,10 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 const uint64_t gi = t.start + e0;
                 const uint64_t o = w * p.d_stride + gi;
                 if (!from_global) cp_async16(slot(it, 0), p.X + o);
-                cp_async16(slot(it, 1), p.opt_m + o);
-                if (kAdamW) cp_async16(slot(it, 2), p.opt_v + o);
+                if (!zero_state) {
+                    cp_async16(slot(it, 1), p.opt_m + o);
+                    if (kAdamW) cp_async16(slot(it, 2), p.opt_v + o);
+                }
                 if (kBf16) cp_async8(slot(it, 3), reinterpret_cast<const __nv_bfloat16*>(p.grad) + o);
                 else cp_async16(slot(it, 3), reinterpret_cast<const float*>(p.grad) + o);
                 if (w == 0) {
@@ -88,8 +95,13 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 } else {
                     take(it, 0, xi);
                 }
-                take(it, 1, mi);
-                if (kAdamW) take(it, 2, vi);
+                if (zero_state) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) mi[j] = vi[j] = 0.f;
+                } else {
+                    take(it, 1, mi);
+                    if (kAdamW) take(it, 2, vi);
+                }
                 if (kBf16) {
                     const uint2 raw = *reinterpret_cast<const uint2*>(slot(it, 3));
                     gr[0] = __uint_as_float(raw.x << 16);
@@ -106,8 +118,10 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                     else sgdm_elem(xi[j], mi[j], gr[j], sa);
                     dif[w][j] = __fsub_rn(x[j], xi[j]);
                 }
-                store4(p.opt_m + o, mi);
-                if (kAdamW) store4(p.opt_v + o, vi);
+                if (keep_state) {
+                    store4(p.opt_m + o, mi);
+                    if (kAdamW) store4(p.opt_v + o, vi);
+                }
                 // refill the slot just read; the arithmetic above consumed its values, so the
                 // shared-memory reads are complete before the asynchronous copy can overwrite them
                 issue(next_issue++);
@@ -142,15 +156,15 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
 #pragma unroll
                 for (int w = 0; w < NW; ++w) {
                     const uint64_t o = w * p.d_stride + gj;
-                    float xi = from_global ? x : p.X[o], mi = p.opt_m[o];
+                    float xi = from_global ? x : p.X[o], mi = zero_state ? 0.f : p.opt_m[o];
                     if (kAdamW) {
-                        float vi = p.opt_v[o];
+                        float vi = zero_state ? 0.f : p.opt_v[o];
                         adamw_elem(xi, mi, vi, load_grad1(p.grad, kBf16, o), a, lam_l);
-                        p.opt_v[o] = vi;
+                        if (keep_state) p.opt_v[o] = vi;
                     } else {
                         sgdm_elem(xi, mi, load_grad1(p.grad, kBf16, o), sa);
                     }
-                    p.opt_m[o] = mi;
+                    if (keep_state) p.opt_m[o] = mi;
                     d[w] = __fsub_rn(x, xi);
                 }
                 float r = 0.f;
@@ -223,12 +237,12 @@ cudaError_t query_fused_shape(const Problem& p, LaunchShape* out) {
 }
 
 cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
-                                     const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s) {
+                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s) {
     if (!fused_round_available(p)) return cudaErrorInvalidValue;
     const int grid = clamp_grid(ls.grid_fused, p.num_tiles);
     if (grid == 0) return cudaSuccess;
     fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, fused_smem_for(p, p.opt_v != nullptr), s>>>(
-        p, a, sa, g, from_x ? 1 : 0);
+        p, a, sa, g, opts);
     return cudaGetLastError();
 }
 

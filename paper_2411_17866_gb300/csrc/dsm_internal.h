@@ -125,15 +125,20 @@ cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t seed_k
                         cudaStream_t s);
 cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s);
 // from_x: every worker starts from the global x (the replicas' reset is pending).
+// zero_state: every worker's base-optimizer state is zero (its reset is pending); none is read.
 cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, bool from_x,
-                               cudaStream_t s);
+                               bool zero_state, cudaStream_t s);
 cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, bool from_x,
-                              cudaStream_t s);
+                              bool zero_state, cudaStream_t s);
 // The fused round's last local step + sign-momentum global step (n <= 8).
+// Options of the fused kernel (bits of its `opts` argument).
+constexpr int kFusedFromX = 1;      // the replicas' reset is pending: every worker starts from x
+constexpr int kFusedZeroState = 2;  // the base-optimizer states are zero: none is read
+constexpr int kFusedDropState = 4;  // the new base-optimizer states are not written (the round resets them)
 bool fused_round_available(const Problem& p);
 cudaError_t query_fused_shape(const Problem& p, LaunchShape* out);  // sets grid_fused (out->sms must be set)
 cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
-                                     const SgdmScalars& sa, const GlobalScalars& g, bool from_x, cudaStream_t s);
+                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s);
 cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);
 cudaError_t launch_stats(const Problem& p, cudaStream_t s);
 

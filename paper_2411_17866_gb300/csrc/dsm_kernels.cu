@@ -152,19 +152,22 @@ __device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t item,
 
 // K2: one AdamW local step on every worker (work item = (worker, tile)),
 // double-buffered in registers.  kFromGlobal: every worker starts from the
-// global x (the replicas' reset is still pending).
-template <bool kBf16, bool kFromGlobal>
+// global x (the replicas' reset is still pending).  kZeroState: the moments
+// are zero (the round restarts the base optimizer) and are not read.
+template <bool kBf16, bool kFromGlobal, bool kZeroState>
 __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars a) {
     const uint32_t items = p.num_tiles * p.n;
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
     LocalItem nx = local_item<kFromGlobal>(p, item, e0, true);
-    float x[4], m[4], v[4], g[4];
+    float x[4], m[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f}, g[4];
     if (nx.vec) {
         load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
-        load4(p.opt_m + nx.base + e0, m);
-        load4(p.opt_v + nx.base + e0, v);
+        if (!kZeroState) {
+            load4(p.opt_m + nx.base + e0, m);
+            load4(p.opt_v + nx.base + e0, v);
+        }
         load4_grad<kBf16>(p.grad, nx.base + e0, g);
     }
     for (; item < items; item += gridDim.x) {
@@ -177,8 +180,10 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
             nx = local_item<kFromGlobal>(p, next, e0, true);
             if (nx.vec) {
                 load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
-                load4(p.opt_m + nx.base + e0, m);
-                load4(p.opt_v + nx.base + e0, v);
+                if (!kZeroState) {
+                    load4(p.opt_m + nx.base + e0, m);
+                    load4(p.opt_v + nx.base + e0, v);
+                }
                 load4_grad<kBf16>(p.grad, nx.base + e0, g);
             }
         }
@@ -192,7 +197,8 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
             const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
                 const uint64_t i = cur.base + e;
-                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i], ms = p.opt_m[i], vs = p.opt_v[i];
+                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i];
+                float ms = kZeroState ? 0.f : p.opt_m[i], vs = kZeroState ? 0.f : p.opt_v[i];
                 adamw_elem(xs, ms, vs, load_grad1(p.grad, kBf16, i), a, cur.lam);
                 p.X[i] = xs; p.opt_m[i] = ms; p.opt_v[i] = vs;
             }
@@ -201,17 +207,18 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
 }
 
 // K3: one SGD-momentum local step on every worker, double-buffered.
-template <bool kBf16, bool kFromGlobal>
+// kFromGlobal, kZeroState: as for K2 (the buffer is zero and not read).
+template <bool kBf16, bool kFromGlobal, bool kZeroState>
 __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars a) {
     const uint32_t items = p.num_tiles * p.n;
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
     LocalItem nx = local_item<kFromGlobal>(p, item, e0, false);
-    float x[4], b[4], g[4];
+    float x[4], b[4] = {0.f, 0.f, 0.f, 0.f}, g[4];
     if (nx.vec) {
         load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
-        load4(p.opt_m + nx.base + e0, b);
+        if (!kZeroState) load4(p.opt_m + nx.base + e0, b);
         load4_grad<kBf16>(p.grad, nx.base + e0, g);
     }
     for (; item < items; item += gridDim.x) {
@@ -224,7 +231,7 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
             nx = local_item<kFromGlobal>(p, next, e0, false);
             if (nx.vec) {
                 load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
-                load4(p.opt_m + nx.base + e0, b);
+                if (!kZeroState) load4(p.opt_m + nx.base + e0, b);
                 load4_grad<kBf16>(p.grad, nx.base + e0, g);
             }
         }
@@ -237,7 +244,7 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
             const uint32_t e1 = min(e0 + kElemsPerThread, cur.len);
             for (uint32_t e = e0; e < e1; ++e) {
                 const uint64_t i = cur.base + e;
-                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i], bs = p.opt_m[i];
+                float xs = kFromGlobal ? p.x[cur.start + e] : p.X[i], bs = kZeroState ? 0.f : p.opt_m[i];
                 sgdm_elem(xs, bs, load_grad1(p.grad, kBf16, i), a);
                 p.X[i] = xs; p.opt_m[i] = bs;
             }
@@ -520,18 +527,20 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     // n = 4: 1.00 of the copy bandwidth with 3, 0.95 with 4); with bf16 gradients 4 are better
     // (GPT-2 M, n = 8: 0.97 with 4, 0.90 with 3; GPT-2 XL, n = 4: 0.96 with 4, 0.87 with 3).
     const int kAdamwCtasPerSm = p.grad_bf16 ? 4 : 3;
-    out->grid_adamw = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, false>, sms)
-                                           : grid_for(k_local_adamw<false, false>, sms), kAdamwCtasPerSm * sms);
+    out->grid_adamw = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, false, false>, sms)
+                                           : grid_for(k_local_adamw<false, false, false>, sms), kAdamwCtasPerSm * sms);
     // The SGD-momentum step fits 6 CTAs per SM, but 4 stream better (GB300, GPT-2 L layout, n = 8:
     // 0.96 of the copy bandwidth with 4, 0.91 with 6, 0.91 with 3), as many as the AdamW step holds.
     constexpr int kSgdmCtasPerSm = 4;
-    out->grid_sgdm = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, false>, sms)
-                                          : grid_for(k_local_sgdm<false, false>, sms), kSgdmCtasPerSm * sms);
+    out->grid_sgdm = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, false, false>, sms)
+                                          : grid_for(k_local_sgdm<false, false, false>, sms), kSgdmCtasPerSm * sms);
     if (fused_round_available(p)) {
-        out->grid_adamw_from_x = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, true>, sms)
-                                                      : grid_for(k_local_adamw<false, true>, sms), kAdamwCtasPerSm * sms);
-        out->grid_sgdm_from_x = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, true>, sms)
-                                                     : grid_for(k_local_sgdm<false, true>, sms), kSgdmCtasPerSm * sms);
+        out->grid_adamw_from_x = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, true, false>, sms)
+                                                      : grid_for(k_local_adamw<false, true, false>, sms),
+                                          kAdamwCtasPerSm * sms);
+        out->grid_sgdm_from_x = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, true, false>, sms)
+                                                     : grid_for(k_local_sgdm<false, true, false>, sms),
+                                         kSgdmCtasPerSm * sms);
         cudaError_t e = query_fused_shape(p, out);
         if (e != cudaSuccess) return e;
     }
@@ -554,33 +563,44 @@ cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const Grad
     return cudaGetLastError();
 }
 
+// The kernel instantiation for (gradient type, from x, zero state).
+using AdamwKernel = void (*)(Problem, AdamScalars);
+using SgdmKernel = void (*)(Problem, SgdmScalars);
+
+static AdamwKernel adamw_kernel_for(bool bf16, bool from_x, bool zero_state) {
+    if (bf16) {
+        if (from_x) return zero_state ? k_local_adamw<true, true, true> : k_local_adamw<true, true, false>;
+        return zero_state ? k_local_adamw<true, false, true> : k_local_adamw<true, false, false>;
+    }
+    if (from_x) return zero_state ? k_local_adamw<false, true, true> : k_local_adamw<false, true, false>;
+    return zero_state ? k_local_adamw<false, false, true> : k_local_adamw<false, false, false>;
+}
+
+static SgdmKernel sgdm_kernel_for(bool bf16, bool from_x, bool zero_state) {
+    if (bf16) {
+        if (from_x) return zero_state ? k_local_sgdm<true, true, true> : k_local_sgdm<true, true, false>;
+        return zero_state ? k_local_sgdm<true, false, true> : k_local_sgdm<true, false, false>;
+    }
+    if (from_x) return zero_state ? k_local_sgdm<false, true, true> : k_local_sgdm<false, true, false>;
+    return zero_state ? k_local_sgdm<false, false, true> : k_local_sgdm<false, false, false>;
+}
+
 cudaError_t launch_local_adamw(const Problem& p, const LaunchShape& ls, const AdamScalars& a, bool from_x,
-                               cudaStream_t s) {
+                               bool zero_state, cudaStream_t s) {
     const uint64_t items = static_cast<uint64_t>(p.num_tiles) * p.n;
+    // the zero-state variants read less and use the grids of the state-reading ones
     const int grid = clamp_grid(from_x ? ls.grid_adamw_from_x : ls.grid_adamw, items);
     if (grid == 0) return cudaSuccess;
-    if (from_x) {
-        if (p.grad_bf16) k_local_adamw<true, true><<<grid, kThreads, 0, s>>>(p, a);
-        else k_local_adamw<false, true><<<grid, kThreads, 0, s>>>(p, a);
-    } else {
-        if (p.grad_bf16) k_local_adamw<true, false><<<grid, kThreads, 0, s>>>(p, a);
-        else k_local_adamw<false, false><<<grid, kThreads, 0, s>>>(p, a);
-    }
+    adamw_kernel_for(p.grad_bf16, from_x, zero_state)<<<grid, kThreads, 0, s>>>(p, a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const SgdmScalars& a, bool from_x,
-                              cudaStream_t s) {
+                              bool zero_state, cudaStream_t s) {
     const uint64_t items = static_cast<uint64_t>(p.num_tiles) * p.n;
     const int grid = clamp_grid(from_x ? ls.grid_sgdm_from_x : ls.grid_sgdm, items);
     if (grid == 0) return cudaSuccess;
-    if (from_x) {
-        if (p.grad_bf16) k_local_sgdm<true, true><<<grid, kThreads, 0, s>>>(p, a);
-        else k_local_sgdm<false, true><<<grid, kThreads, 0, s>>>(p, a);
-    } else {
-        if (p.grad_bf16) k_local_sgdm<true, false><<<grid, kThreads, 0, s>>>(p, a);
-        else k_local_sgdm<false, false><<<grid, kThreads, 0, s>>>(p, a);
-    }
+    sgdm_kernel_for(p.grad_bf16, from_x, zero_state)<<<grid, kThreads, 0, s>>>(p, a);
     return cudaGetLastError();
 }
 

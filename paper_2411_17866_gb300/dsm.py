@@ -26,6 +26,7 @@ F32, BF16 = 0, 1
 BUF_X, BUF_M, BUF_REPLICA, BUF_OPT_M, BUF_OPT_V, BUF_GRAD, BUF_GLOBAL_V = 0, 1, 2, 3, 4, 5, 6
 GLOBAL_SIGN_MOMENTUM, GLOBAL_SLOWMO, GLOBAL_SIGNED_SLOWMO, GLOBAL_LOOKAHEAD, GLOBAL_ADAMW = 0, 1, 2, 3, 4
 FLAG_FUSED_ROUND = 1
+FLAG_RESET_LOCAL_STATE = 2
 
 ERROR_NAMES = {DSM_EINVAL: "DSM_EINVAL", DSM_ENOMEM: "DSM_ENOMEM", DSM_EALIGN: "DSM_EALIGN",
                DSM_ESTATE: "DSM_ESTATE", DSM_ECUDA: "DSM_ECUDA", DSM_ERANGE: "DSM_ERANGE"}

@@ -75,6 +75,7 @@ def test_state_bytes_covers_the_state(lib):
     (dict(hp=W.HParams(sign_mode=3)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(sign_mode=W.RSIGN_ZERO, rsign_B=0.0)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(grad_dtype=2)), dsm.DSM_EINVAL),
+    (dict(hp=W.HParams(flags=4)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(base=7)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(global_mode=5)), dsm.DSM_EINVAL),
     (dict(hp=W.HParams(global_mode=W.GLOBAL_SLOWMO, sign_mode=W.RSIGN_ZERO)), dsm.DSM_EINVAL),
@@ -94,6 +95,13 @@ def test_invalid_arguments_are_rejected(lib, bad, code):
     assert rc == code, dsm.last_error()
     assert h.value is None
     assert dsm.last_error()
+
+
+def test_known_flags_are_accepted(lib):
+    for flags in (W.FLAG_FUSED_ROUND, W.FLAG_RESET_LOCAL_STATE, W.FLAG_FUSED_ROUND | W.FLAG_RESET_LOCAL_STATE):
+        lay, n, hp = _args(hp=W.HParams(flags=flags))
+        assert dsm.dsm_state_bytes(lay, n, hp) > 0
+    assert (dsm.FLAG_FUSED_ROUND, dsm.FLAG_RESET_LOCAL_STATE) == (W.FLAG_FUSED_ROUND, W.FLAG_RESET_LOCAL_STATE)
 
 
 def test_arena_checks(lib):

@@ -456,3 +456,90 @@ def test_state_dict_round_trip(fused):
         assert torch.equal(a.read(which, w), b.read(which, w))
     a.close()
     b.close()
+
+
+RESET = [
+    ("adamw-f32-n4-t3", ADAMW, 4, 3),
+    ("adamw-bf16-n3-t1", dataclasses.replace(ADAMW, grad_dtype=W.BF16, seed=5), 3, 1),
+    ("sgdm-rsign-n8-t2", SGDM, 8, 2),
+    ("sgdm-bf16-n2-t1", dataclasses.replace(SGDM, grad_dtype=W.BF16, sign_mode=W.SIGN), 2, 1),
+    ("adamw-n9-generic-t2", ADAMW, 9, 2),
+    ("slowmo-adamw-n4-t2", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO, g_b1=0.5, g_eta=0.8), 4, 2),
+    ("global-adamw-n3-t2", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_ADAMW), 3, 2),
+]
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+@pytest.mark.parametrize("layout_name", ["ragged", "mini"])
+@pytest.mark.parametrize("name,hp,n,tau", RESET, ids=[c[0] for c in RESET])
+def test_reset_local_state_bitexact(layout_name, name, hp, n, tau, fused):
+    """Every round restarts each worker's base optimizer (zero state, AdamW count j = k + 1): three
+    rounds against the oracle, the states read back mid-round (the restarted optimizer's values) and
+    between rounds (zeros)."""
+    tensors = RAGGED if layout_name == "ragged" else MINI
+    flags = W.FLAG_RESET_LOCAL_STATE | (W.FLAG_FUSED_ROUND if fused else 0)
+    hp = dataclasses.replace(hp, flags=flags)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    for t in range(3):
+        if t == 1:   # mid-round: the first local step restarted from zero state
+            run.fill_synthetic_grads(t * tau)
+            run.local_step()
+            ora.local_step()
+            compare_state(run, ora)
+            for k in range(1, tau):
+                run.fill_synthetic_grads(t * tau + k)
+                run.local_step()
+                ora.local_step()
+            stats = run.global_step(with_stats=True)
+            ora.global_step()
+        else:
+            stats = run.synthetic_round(with_stats=True)
+            ora.run_round()
+        compare_state(run, ora)   # states between rounds: zeros on both sides
+        compare_stats(stats, ora.last_stats, n)
+        assert all(not np.any(o) for o in ora.opt_m)
+    run.close()
+
+
+def test_reset_local_state_differs_from_persistent_state():
+    """The flag changes the method (not only its execution): after two rounds the models differ."""
+    tensors, n, tau = MINI, 2, 2
+    xs = []
+    for flags in (0, W.FLAG_RESET_LOCAL_STATE):
+        run = dsm.DistributedSignMomentum(tensors, n, tau, dataclasses.replace(ADAMW, flags=flags))
+        for _ in range(2):
+            run.synthetic_round()
+        xs.append(run.read(dsm.BUF_X))
+        run.close()
+    assert not torch.equal(xs[0], xs[1])
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+def test_reset_local_state_checkpoint_and_partial_writes(fused):
+    """With the restart pending: a partial write of a state buffer keeps the rest at zero, a checkpoint
+    restores into a fresh handle, and both continue identically to the oracle."""
+    tensors, n, tau = RAGGED, 3, 2
+    flags = W.FLAG_RESET_LOCAL_STATE | (W.FLAG_FUSED_ROUND if fused else 0)
+    hp = dataclasses.replace(ADAMW, flags=flags)
+    a = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp)
+    a.synthetic_round()
+    ora.run_round()
+    st = a.state_dict()
+    assert all(not torch.any(v) for v in st["opt_m"] + st["opt_v"])
+    # a partial write into worker 1's first moment: the oracle gets the same values, the rest stays 0
+    patch = torch.full((100,), 1e-4, dtype=torch.float32)
+    a.write(dsm.BUF_OPT_M, patch, worker=1, offset=50)
+    ora.opt_m[1][50:150] = patch.numpy()
+    compare_state(a, ora)
+    b = dsm.DistributedSignMomentum(tensors, n, tau, hp, x0=torch.zeros(a.d))
+    b.load_state_dict(a.state_dict())
+    for _ in range(2):
+        a.synthetic_round()
+        b.synthetic_round()
+        ora.run_round()
+    compare_state(a, ora)
+    compare_state(b, ora)
+    a.close()
+    b.close()
