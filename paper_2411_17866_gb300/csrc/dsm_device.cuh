@@ -354,9 +354,9 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 
 // Persistent grid: every SM times the CTAs of `kernel` that fit on one SM.
 template <typename K>
-int grid_for(K kernel, int sms, size_t smem = 0) {
+int grid_for(K kernel, int sms, size_t smem = 0, int threads = kThreads) {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem) != cudaSuccess || per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem) != cudaSuccess || per_sm < 1)
         per_sm = 1;
     return sms * per_sm;
 }

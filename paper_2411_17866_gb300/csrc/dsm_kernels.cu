@@ -19,6 +19,7 @@
 // paper's expression evaluated one operation at a time.
 
 #include <algorithm>
+#include <type_traits>
 
 #include "dsm_device.cuh"
 
@@ -57,62 +58,94 @@ __global__ void __launch_bounds__(kThreads) k_init(Problem p, uint64_t key_init,
 
 // K1: synthetic gradients of one local step for every worker.  Bound by the
 // integer work of the hash (one 64-bit SplitMix64 output per two elements
-// and per draw family), not by its write stream.
-template <bool kBf16, bool kPrescaled>
-__device__ __forceinline__ void grad_fill4(const Problem& p, const GradKeys& k, uint64_t gi, float s, float s2) {
-    // even gi: elements gi..gi+3 use outputs gi/2+1, gi/2+2; output j of any
-    // family is finalise(key + j*gamma), and j*gamma is shared by all families
-    const uint64_t jg0 = ((gi >> 1) + 1) * kGoldenGamma, jg1 = jg0 + kGoldenGamma;
-    const uint64_t h0 = sm64_finalise(k.step + jg0), h1 = sm64_finalise(k.step + jg1);
-    float a[4];
-    if (kPrescaled) {
-        a[0] = __fmul_rn(s, centred_even(h0)); a[1] = __fmul_rn(s, centred_odd(h0));
-        a[2] = __fmul_rn(s, centred_even(h1)); a[3] = __fmul_rn(s, centred_odd(h1));
-    } else {
-        a[0] = step_term(s, draw_even(h0)); a[1] = step_term(s, draw_odd(h0));
-        a[2] = step_term(s, draw_even(h1)); a[3] = step_term(s, draw_odd(h1));
-    }
-    for (uint32_t w = 0; w < p.n; ++w) {
-        const uint64_t q0 = sm64_finalise(k.worker[w] + jg0), q1 = sm64_finalise(k.worker[w] + jg1);
-        float g[4];
+// and per draw family), not by its write stream.  A CTA of kFillThreads
+// threads fills one tile; a thread owns kFillGroups groups of 4 elements
+// (group q at 4*thread + q*4*kFillThreads), so it carries 2*kFillGroups
+// independent hash chains per family, and every warp store covers 512
+// contiguous bytes of fp32 (256 of bf16).
+constexpr uint32_t kFillThreads = 64;
+constexpr uint32_t kFillGroups = kTile / (4 * kFillThreads);  // 4
+
+// Output j of any family is finalise(key + j*gamma); the j*gamma of a
+// group (j = e/2 + 1 and e/2 + 2 for its even first element e) is shared by
+// the step family and every worker family.
+template <bool kBf16, bool kPrescaled, int kGroups, uint32_t kGroupStride>
+__device__ __forceinline__ void grad_fill_groups(const Problem& p, const GradKeys& k, uint64_t gi0, float s,
+                                                 float s2) {
+    uint64_t jg0[kGroups], jg1[kGroups];
+    float a[kGroups][4];
+#pragma unroll
+    for (int q = 0; q < kGroups; ++q) {
+        const uint64_t gi = gi0 + q * kGroupStride;
+        jg0[q] = ((gi >> 1) + 1) * kGoldenGamma;
+        jg1[q] = jg0[q] + kGoldenGamma;
+        const uint64_t h0 = sm64_finalise(k.step + jg0[q]), h1 = sm64_finalise(k.step + jg1[q]);
         if (kPrescaled) {
-            g[0] = __fadd_rn(a[0], __fmul_rn(s2, centred_even(q0)));
-            g[1] = __fadd_rn(a[1], __fmul_rn(s2, centred_odd(q0)));
-            g[2] = __fadd_rn(a[2], __fmul_rn(s2, centred_even(q1)));
-            g[3] = __fadd_rn(a[3], __fmul_rn(s2, centred_odd(q1)));
+            a[q][0] = __fmul_rn(s, centred_even(h0)); a[q][1] = __fmul_rn(s, centred_odd(h0));
+            a[q][2] = __fmul_rn(s, centred_even(h1)); a[q][3] = __fmul_rn(s, centred_odd(h1));
         } else {
-            g[0] = grad_value(a[0], s2, draw_even(q0)); g[1] = grad_value(a[1], s2, draw_odd(q0));
-            g[2] = grad_value(a[2], s2, draw_even(q1)); g[3] = grad_value(a[3], s2, draw_odd(q1));
+            a[q][0] = step_term(s, draw_even(h0)); a[q][1] = step_term(s, draw_odd(h0));
+            a[q][2] = step_term(s, draw_even(h1)); a[q][3] = step_term(s, draw_odd(h1));
         }
+    }
+    using Elem = typename std::conditional<kBf16, __nv_bfloat16, float>::type;
+    Elem* out = reinterpret_cast<Elem*>(p.grad) + gi0;
+    for (uint32_t w = 0; w < p.n; ++w, out += p.d_stride) {
+#pragma unroll
+        for (int q = 0; q < kGroups; ++q) {
+            const uint64_t q0 = sm64_finalise(k.worker[w] + jg0[q]), q1 = sm64_finalise(k.worker[w] + jg1[q]);
+            float g[4];
+            if (kPrescaled) {
+                g[0] = __fadd_rn(a[q][0], __fmul_rn(s2, centred_even(q0)));
+                g[1] = __fadd_rn(a[q][1], __fmul_rn(s2, centred_odd(q0)));
+                g[2] = __fadd_rn(a[q][2], __fmul_rn(s2, centred_even(q1)));
+                g[3] = __fadd_rn(a[q][3], __fmul_rn(s2, centred_odd(q1)));
+            } else {
+                g[0] = grad_value(a[q][0], s2, draw_even(q0)); g[1] = grad_value(a[q][1], s2, draw_odd(q0));
+                g[2] = grad_value(a[q][2], s2, draw_even(q1)); g[3] = grad_value(a[q][3], s2, draw_odd(q1));
+            }
+            if (kBf16) store4_bf16(reinterpret_cast<__nv_bfloat16*>(out) + q * kGroupStride, g);
+            else store4(reinterpret_cast<float*>(out) + q * kGroupStride, g);
+        }
+    }
+}
+
+// Element-by-element fill (tile starts that are not 4-aligned, ragged tails).
+template <bool kBf16>
+__device__ __forceinline__ void grad_fill_elem(const Problem& p, const GradKeys& k, uint64_t gi, float s, float s2) {
+    const float a = step_term(s, hash_uniform(k.step, gi));
+    for (uint32_t w = 0; w < p.n; ++w) {
+        const float g = grad_value(a, s2, hash_uniform(k.worker[w], gi));
         const uint64_t o = w * p.d_stride + gi;
-        if (kBf16) store4_bf16(reinterpret_cast<__nv_bfloat16*>(p.grad) + o, g);
-        else store4(reinterpret_cast<float*>(p.grad) + o, g);
+        if (kBf16) reinterpret_cast<__nv_bfloat16*>(p.grad)[o] = __float2bfloat16_rn(g);
+        else reinterpret_cast<float*>(p.grad)[o] = g;
     }
 }
 
 template <bool kBf16>
-__global__ void __launch_bounds__(kThreads) k_grad_fill(Problem p, GradKeys k) {
-    const uint32_t e0 = threadIdx.x * kElemsPerThread;
+__global__ void __launch_bounds__(kFillThreads) k_grad_fill(Problem p, GradKeys k) {
+    constexpr uint32_t kStride = 4 * kFillThreads;  // elements between a thread's groups
     for (uint32_t ti = blockIdx.x; ti < p.num_tiles; ti += gridDim.x) {
         const TileDesc td = p.tiles[ti];
         const TensorDesc& T = p.tensors[td.tensor];
         const float s = T.scale, s2 = T.scale2;
-        if (vector_ok(td, e0)) {
-            if (fabsf(s) >= kMinPrescaled && fabsf(s2) >= kMinPrescaled)
-                grad_fill4<kBf16, true>(p, k, td.start + e0, __fmul_rn(s, kTwoPowM24), __fmul_rn(s2, kTwoPowM24));
-            else
-                grad_fill4<kBf16, false>(p, k, td.start + e0, s, s2);
-        } else {
-            const uint32_t e1 = min(e0 + kElemsPerThread, td.len);
-            for (uint32_t e = e0; e < e1; ++e) {
-                const uint64_t gi = td.start + e;
-                const float a = step_term(s, hash_uniform(k.step, gi));
-                for (uint32_t w = 0; w < p.n; ++w) {
-                    const float g = grad_value(a, s2, hash_uniform(k.worker[w], gi));
-                    const uint64_t o = w * p.d_stride + gi;
-                    if (kBf16) reinterpret_cast<__nv_bfloat16*>(p.grad)[o] = __float2bfloat16_rn(g);
-                    else reinterpret_cast<float*>(p.grad)[o] = g;
-                }
+        // one multiplication per draw where both scales allow it (see centred_even)
+        const bool pre = fabsf(s) >= kMinPrescaled && fabsf(s2) >= kMinPrescaled;
+        const float sp = __fmul_rn(s, kTwoPowM24), sp2 = __fmul_rn(s2, kTwoPowM24);
+        const bool aligned = (td.start & 3u) == 0;
+        if (aligned && td.len == kTile) {  // a full tile (uniform across the CTA)
+            const uint64_t gi0 = td.start + threadIdx.x * 4;
+            if (pre) grad_fill_groups<kBf16, true, kFillGroups, kStride>(p, k, gi0, sp, sp2);
+            else grad_fill_groups<kBf16, false, kFillGroups, kStride>(p, k, gi0, s, s2);
+            continue;
+        }
+        for (uint32_t e0 = threadIdx.x * 4; e0 < td.len; e0 += kStride) {  // a ragged tile, group by group
+            if (aligned && e0 + 4 <= td.len) {
+                if (pre) grad_fill_groups<kBf16, true, 1, kStride>(p, k, td.start + e0, sp, sp2);
+                else grad_fill_groups<kBf16, false, 1, kStride>(p, k, td.start + e0, s, s2);
+            } else {
+                const uint32_t e1 = min(e0 + 4u, td.len);
+                for (uint32_t e = e0; e < e1; ++e) grad_fill_elem<kBf16>(p, k, td.start + e, s, s2);
             }
         }
     }
@@ -522,7 +555,8 @@ cudaError_t query_launch_shape(const Problem& p, LaunchShape* out) {
     if (err != cudaSuccess) return err;
     out->sms = sms;
     out->grid_init = grid_for(k_init, sms);
-    out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms) : grid_for(k_grad_fill<false>, sms);
+    out->grid_grad = p.grad_bf16 ? grid_for(k_grad_fill<true>, sms, 0, kFillThreads)
+                                 : grid_for(k_grad_fill<false>, sms, 0, kFillThreads);
     // The AdamW step fits 4 CTAs per SM.  With fp32 gradients it streams better with 3 (GB300, GPT-2 S,
     // n = 4: 1.00 of the copy bandwidth with 3, 0.95 with 4); with bf16 gradients 4 are better
     // (GPT-2 M, n = 8: 0.97 with 4, 0.90 with 3; GPT-2 XL, n = 4: 0.96 with 4, 0.87 with 3).
@@ -558,8 +592,8 @@ cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t key_in
 cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s) {
     const int grid = clamp_grid(ls.grid_grad, p.num_tiles);
     if (grid == 0) return cudaSuccess;
-    if (p.grad_bf16) k_grad_fill<true><<<grid, kThreads, 0, s>>>(p, k);
-    else k_grad_fill<false><<<grid, kThreads, 0, s>>>(p, k);
+    if (p.grad_bf16) k_grad_fill<true><<<grid, kFillThreads, 0, s>>>(p, k);
+    else k_grad_fill<false><<<grid, kFillThreads, 0, s>>>(p, k);
     return cudaGetLastError();
 }
 
