@@ -424,22 +424,24 @@ def main():
         for i in range(wl.n):
             run.read(dsm.BUF_GRAD, i, out=host_g[i], stream=stream)
         host_x = torch.empty(wl.d, dtype=torch.float32).pin_memory()
+        copy_stream = torch.cuda.Stream(dev)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         t0 = time.perf_counter()
         for _ in range(args.e2e_steps):
             for k in range(tau):
-                run.load_grads(host_g, stream)
-                run.local_step(stream)
+                # the copy of each chunk of gradients overlaps the update of the previous chunk
+                run.local_step_host_grads(host_g, stream, copy_stream)
             run.global_step(stream)
             run.read(dsm.BUF_X, out=host_x, stream=stream)   # synchronises the stream
             t += 1
         e2e_dt = max_over_ranks(time.perf_counter() - t0, world)
         e2e = {"value": whole_job_value(wl.d, world, args.e2e_steps, e2e_dt), "unit": UNIT,
                "h2d_bytes_per_step": tau * wl.n * wl.d * esz, "d2h_bytes_per_step": wl.d * 4,
-               "steps": args.e2e_steps, "path": "dsm_load_grads (pinned host) + dsm_local_step x tau, "
-                                                 "dsm_global_step, dsm_read_params(x -> pinned host)"}
+               "steps": args.e2e_steps, "path": "dsm_local_step_host_grads (pinned host gradients, chunked "
+                                                 "copies on a second stream) x tau, dsm_global_step, "
+                                                 "dsm_read_params(x -> pinned host)"}
 
     if rank != 0:
         if world > 1:

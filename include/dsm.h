@@ -259,6 +259,30 @@ int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream
  * if tau local steps were already done in this round.  Asynchronous. */
 int dsm_local_step(dsm_handle* h, dsm_stream_t stream);
 
+/* Local step k of the current round, Eq. (local-steps), with the gradients
+ * of every worker (the grad f_i of Eq. (base-sgd)) taken from host memory,
+ * and their transfer overlapped with the update.  src is a dense [n][d]
+ * array of the gradient type in host memory, the caller's; pinned memory
+ * makes the copies asynchronous (pageable memory works, without overlap).
+ * The model is cut into chunks of whole tiles (about 64 MB of gradients
+ * each, at most 64): for every chunk the call enqueues the copy of its n
+ * gradient slices on copy_stream and, on stream, the local step on that
+ * chunk once its copy has landed, so that the copy of one chunk runs while
+ * the previous chunk is updated.  The copies start after everything
+ * enqueued on stream before the call; work enqueued on stream after the
+ * call follows every copy and every update.  copy_stream may equal stream
+ * (no overlap).  Same results, bit for bit, as dsm_load_grads followed by
+ * dsm_local_step; with the fused round's last step the copies are enqueued
+ * and the update is left to dsm_global_step, as for dsm_local_step.  The
+ * first call creates the handle's chunk events (cudaEventCreate); the
+ * environment variable DSM_HOST_GRAD_CHUNK_BYTES, read then, sets another
+ * chunk size.  src must stay unchanged until the copies have completed (until
+ * stream reaches work enqueued after the call).
+ * DSM_EINVAL for NULL handle or src, DSM_ESTATE as for dsm_local_step,
+ * DSM_ECUDA if an event, copy or launch fails to enqueue (the step is then
+ * not counted, and the gradients and states are undefined). */
+int dsm_local_step_host_grads(dsm_handle* h, const void* src, dsm_stream_t stream, dsm_stream_t copy_stream);
+
 /* Global step of Algorithm 1 after the round's tau local steps (else
  * DSM_ESTATE): Delta = (1/n) sum_{i=0..n-1} (x - x_i) (summed in worker
  * order), u = b1 m + ((1-b1)/gamma) Delta, x' = x - eta gamma (S(u) + lambda x),

@@ -197,6 +197,15 @@ struct dsm_handle {
     AdamScalars pending_a{};
     SgdmScalars pending_sa{};
     uint64_t j = 0;        // AdamW step count of the last local step (restarts each round with the reset flag)
+    // local steps with host gradients (dsm_local_step_host_grads): chunk c covers tiles
+    // [chunk_tile[c], chunk_tile[c+1]); ev_copied[c] marks its gradients in the arena
+    std::vector<uint32_t> chunk_tile;
+    std::vector<cudaEvent_t> ev_copied;
+    cudaEvent_t ev_entry = nullptr;  // the caller's stream at entry (every earlier reader or writer)
+    ~dsm_handle() {
+        for (cudaEvent_t e : ev_copied) cudaEventDestroy(e);
+        if (ev_entry) cudaEventDestroy(ev_entry);
+    }
 };
 
 namespace {
@@ -266,12 +275,51 @@ void next_local_scalars(const dsm_handle* h, AdamScalars* a, SgdmScalars* sa, do
     }
 }
 
-cudaError_t launch_local(dsm_handle* h, const AdamScalars& a, const SgdmScalars& sa, cudaStream_t s) {
+// The local step on the tiles of problem q (the whole model, or a chunk of it).
+cudaError_t launch_local_on(const dsm_handle* h, const Problem& q, const AdamScalars& a, const SgdmScalars& sa,
+                            cudaStream_t s) {
     const bool from_x = h->replicas_stale, zero_state = h->states_zero;
-    cudaError_t err = h->hp.base == DSM_BASE_ADAMW ? launch_local_adamw(h->prob, h->shape, a, from_x, zero_state, s)
-                                                   : launch_local_sgdm(h->prob, h->shape, sa, from_x, zero_state, s);
+    return h->hp.base == DSM_BASE_ADAMW ? launch_local_adamw(q, h->shape, a, from_x, zero_state, s)
+                                        : launch_local_sgdm(q, h->shape, sa, from_x, zero_state, s);
+}
+
+cudaError_t launch_local(dsm_handle* h, const AdamScalars& a, const SgdmScalars& sa, cudaStream_t s) {
+    cudaError_t err = launch_local_on(h, h->prob, a, sa, s);
     if (err == cudaSuccess) h->replicas_stale = h->states_zero = false;
     return err;
+}
+
+// Chunks of whole tiles for dsm_local_step_host_grads: about kChunkBytes of gradients (all
+// workers) each, at most kMaxChunks, and their events (created on first use).
+constexpr uint64_t kChunkBytes = 64ull << 20;
+constexpr uint32_t kMaxChunks = 64;
+
+int prepare_chunks(dsm_handle* h) {
+    if (!h->chunk_tile.empty()) return DSM_OK;
+    const uint64_t grad_bytes = uint64_t(h->n) * h->al.d * h->al.grad_esize;
+    uint64_t chunk_bytes = kChunkBytes;
+    if (const char* env = std::getenv("DSM_HOST_GRAD_CHUNK_BYTES")) {  // a different chunk size (tests, tuning)
+        const unsigned long long v = std::strtoull(env, nullptr, 10);
+        if (v > 0) chunk_bytes = v;
+    }
+    uint64_t c = (grad_bytes + chunk_bytes - 1) / chunk_bytes;
+    c = c < 1 ? 1 : (c > kMaxChunks ? kMaxChunks : c);
+    if (c > h->al.num_tiles) c = h->al.num_tiles;
+    std::vector<cudaEvent_t> ev(c, nullptr);
+    cudaError_t err = cudaSuccess;
+    for (uint64_t i = 0; i < c && err == cudaSuccess; ++i) err = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
+    cudaEvent_t entry = nullptr;
+    if (err == cudaSuccess) err = cudaEventCreateWithFlags(&entry, cudaEventDisableTiming);
+    if (err != cudaSuccess) {
+        for (cudaEvent_t e : ev)
+            if (e) cudaEventDestroy(e);
+        return cuda_fail(err, "create the events of the host-gradient chunks");
+    }
+    h->ev_copied = std::move(ev);
+    h->ev_entry = entry;
+    h->chunk_tile.resize(c + 1);
+    for (uint64_t i = 0; i <= c; ++i) h->chunk_tile[i] = static_cast<uint32_t>(uint64_t(h->al.num_tiles) * i / c);
+    return DSM_OK;
 }
 
 // Runs a deferred last local step unfused (before its inputs or outputs are touched).
@@ -516,6 +564,60 @@ int dsm_local_step(dsm_handle* h, dsm_stream_t stream) {
     return DSM_OK;
 }
 
+int dsm_local_step_host_grads(dsm_handle* h, const void* src, dsm_stream_t stream, dsm_stream_t copy_stream) {
+    if (!h || !src) return fail(DSM_EINVAL, "NULL argument");
+    if (h->k >= h->tau)
+        return fail(DSM_ESTATE, "all %u local steps of round %llu are done; call dsm_global_step", h->tau,
+                    (unsigned long long)h->t);
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaStream_t s = S(stream), cs = S(copy_stream);
+    int rc = prepare_chunks(h);
+    if (rc != DSM_OK) return rc;
+    AdamScalars a;
+    SgdmScalars sa;
+    double nb1, nb2;
+    next_local_scalars(h, &a, &sa, &nb1, &nb2);
+    const bool defer = h->fused && h->k + 1 == h->tau;  // the update runs inside dsm_global_step
+    const size_t es = h->al.grad_esize;
+    char* grad = static_cast<char*>(h->prob.grad);
+    const char* host = static_cast<const char*>(src);
+    // the copies follow everything already enqueued on the caller's stream (earlier readers and
+    // writers of the gradient buffers)
+    cudaError_t err = cudaEventRecord(h->ev_entry, s);
+    if (err == cudaSuccess) err = cudaStreamWaitEvent(cs, h->ev_entry, 0);
+    if (err != cudaSuccess) return cuda_fail(err, "order the gradient copies after the stream");
+    const uint32_t chunks = static_cast<uint32_t>(h->ev_copied.size());
+    for (uint32_t c = 0; c < chunks; ++c) {
+        const uint32_t t0 = h->chunk_tile[c], t1 = h->chunk_tile[c + 1];
+        const uint64_t e0 = h->tiles[t0].start, e1 = h->tiles[t1 - 1].start + h->tiles[t1 - 1].len;
+        err = cudaMemcpy2DAsync(grad + e0 * es, h->al.d_stride * es, host + e0 * es, h->al.d * es, (e1 - e0) * es,
+                                h->n, cudaMemcpyHostToDevice, cs);
+        if (err == cudaSuccess) err = cudaEventRecord(h->ev_copied[c], cs);
+        if (err == cudaSuccess) err = cudaStreamWaitEvent(s, h->ev_copied[c], 0);
+        if (err != cudaSuccess) return cuda_fail(err, "copy a chunk of gradients");
+        if (!defer) {
+            Problem q = h->prob;
+            q.tiles = h->prob.tiles + t0;
+            q.num_tiles = t1 - t0;
+            err = launch_local_on(h, q, a, sa, s);
+            if (err != cudaSuccess) return cuda_fail(err, "launch the local step on a chunk");
+        }
+    }
+    if (defer) {
+        h->pending_a = a;
+        h->pending_sa = sa;
+        h->last_pending = true;
+    } else {
+        h->replicas_stale = h->states_zero = false;
+    }
+    h->b1_pow = nb1;
+    h->b2_pow = nb2;
+    h->j += 1;
+    h->k += 1;
+    return DSM_OK;
+}
+
 int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats, uint32_t stats_count) {
     if (!h) return fail(DSM_EINVAL, "handle is NULL");
     if (h->k != h->tau)
@@ -723,6 +825,8 @@ int dsm_get_info(const dsm_handle* h, dsm_info* out) {
 }
 
 int dsm_destroy(dsm_handle* h) {
+    if (!h) return DSM_OK;
+    DeviceGuard guard(h->device);  // the handle's events belong to its device
     delete h;
     return DSM_OK;
 }

@@ -77,6 +77,7 @@ _PROTOS = {
     "dsm_grad_ptr": (c_int, [c_void_p, c_uint32, POINTER(c_void_p)]),
     "dsm_load_grads": (c_int, [c_void_p, c_void_p, c_int, c_void_p]),
     "dsm_local_step": (c_int, [c_void_p, c_void_p]),
+    "dsm_local_step_host_grads": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
     "dsm_global_step": (c_int, [c_void_p, c_void_p, POINTER(dsm_tensor_stats), c_uint32]),
     "dsm_stats_ptr": (c_int, [c_void_p, POINTER(c_void_p)]),
     "dsm_read_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
@@ -194,6 +195,13 @@ def dsm_load_grads(h, src_ptr: int, src_is_device: bool, stream=None) -> None:
 
 def dsm_local_step(h, stream=None) -> None:
     _check(load_library().dsm_local_step(h, _stream(stream)), "dsm_local_step")
+
+
+def dsm_local_step_host_grads(h, src_ptr: int, stream=None, copy_stream=None) -> None:
+    """``copy_stream``: the stream for the chunked host-to-device copies (None: ``stream``)."""
+    cs = _stream(stream) if copy_stream is None else _stream(copy_stream)
+    _check(load_library().dsm_local_step_host_grads(h, c_void_p(src_ptr), _stream(stream), cs),
+           "dsm_local_step_host_grads")
 
 
 def dsm_global_step(h, stream=None, stats=None) -> None:
@@ -314,6 +322,15 @@ class DistributedSignMomentum:
 
     def local_step(self, stream=None):
         dsm_local_step(self.h, stream)
+
+    def local_step_host_grads(self, src, stream=None, copy_stream=None):
+        """One local step on gradients in host memory (``src``: [n, d] CPU tensor of the gradient type,
+        pinned for overlap), the copy of each chunk overlapped with the update of the previous one."""
+        esize = 2 if self.hp.grad_dtype == BF16 else 4
+        if src.is_cuda or not src.is_contiguous() or tuple(src.shape) != (self.n, self.d) or \
+                src.element_size() != esize:
+            raise ValueError(f"src must be a contiguous [n, d] host tensor of {esize}-byte gradients")
+        dsm_local_step_host_grads(self.h, src.data_ptr(), stream, copy_stream)
 
     def global_step(self, stream=None, with_stats=False):
         if not with_stats:

@@ -7,6 +7,7 @@ be identical bit for bit.  The statistics' sums are compared to a relative
 (n + 4) * 2^-24 (derived in gpu_common.stats_rtol); their counts exactly.
 """
 import dataclasses
+import zlib
 
 import numpy as np
 import pytest
@@ -543,3 +544,76 @@ def test_reset_local_state_checkpoint_and_partial_writes(fused):
     compare_state(b, ora)
     a.close()
     b.close()
+
+
+HOST_GRADS = [
+    ("adamw-f32-n3-t2-fused", dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND), 3, 2),
+    ("adamw-bf16-n8-t2", dataclasses.replace(ADAMW, grad_dtype=W.BF16), 8, 2),
+    ("sgdm-n4-t1-fused", dataclasses.replace(SGDM, flags=W.FLAG_FUSED_ROUND), 4, 1),
+    ("adamw-n9-generic-t2", ADAMW, 9, 2),
+    ("reset-adamw-n4-t3-fused", dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND | W.FLAG_RESET_LOCAL_STATE), 4, 3),
+]
+
+
+@pytest.mark.parametrize("chunk_bytes", ["default", "4096"])
+@pytest.mark.parametrize("layout_name", ["ragged", "mini"])
+@pytest.mark.parametrize("name,hp,n,tau", HOST_GRADS, ids=[c[0] for c in HOST_GRADS])
+def test_host_gradient_steps_bitexact(layout_name, name, hp, n, tau, chunk_bytes, monkeypatch):
+    """dsm_local_step_host_grads: gradients from pinned host memory, copied chunk by chunk on a second
+    stream while the previous chunk is updated; three rounds against the oracle fed the same gradients.
+    A 4096-byte chunk size cuts the model into many chunks, with boundaries inside tensors."""
+    if chunk_bytes != "default":
+        monkeypatch.setenv("DSM_HOST_GRAD_CHUNK_BYTES", chunk_bytes)
+    tensors = RAGGED if layout_name == "ragged" else MINI
+    d = sum(t.numel for t in tensors)
+    rng = np.random.default_rng(zlib.crc32(name.encode()))
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp, with_stats=True)
+    stream = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream()
+    bf16 = hp.grad_dtype == W.BF16
+    keep = []
+    for t in range(3):
+        for k in range(tau):
+            g = torch.from_numpy((rng.standard_normal((n, d)) * 1e-3).astype(np.float32))
+            if bf16:
+                g = g.to(torch.bfloat16)
+            src = g.pin_memory()
+            keep.append(src)   # unchanged until the copies complete
+            run.local_step_host_grads(src, stream, copy_stream)
+            ora.local_step([g[i].to(torch.float32).numpy() for i in range(n)])
+        stats = run.global_step(stream, with_stats=True)
+        ora.global_step()
+        compare_state(run, ora, grads=False)
+        compare_stats(stats, ora.last_stats, n)
+    run.close()
+
+
+def test_host_gradient_steps_mix_with_device_fills():
+    """Host-gradient steps interleaved with synthetic fills and plain local steps on the same handle."""
+    tensors, n, tau = RAGGED, 3, 3
+    hp = dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND)
+    d = sum(t.numel for t in tensors)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp)
+    copy_stream = torch.cuda.Stream()
+    rng = np.random.default_rng(4)
+    keep = []
+    for t in range(2):
+        for k in range(tau):
+            if k == 1:
+                run.fill_synthetic_grads(t * tau + k)
+                run.local_step()
+                ora.local_step()
+            else:
+                g = (rng.standard_normal((n, d)) * 1e-3).astype(np.float32)
+                src = torch.from_numpy(g).pin_memory()
+                keep.append(src)
+                run.local_step_host_grads(src, copy_stream=copy_stream)
+                ora.local_step([g[i] for i in range(n)])
+        run.global_step()
+        ora.global_step()
+    compare_state(run, ora)
+    with pytest.raises(ValueError):
+        run.local_step_host_grads(torch.zeros((n, d + 1)))
+    run.close()
