@@ -159,16 +159,17 @@ def bytes_per_param_global(wl) -> int:
 
 
 def fused_round_active(wl) -> bool:
-    """The library fuses the round for every global step but global AdamW, with n <= 8."""
-    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.hp.global_mode != W.GLOBAL_ADAMW and wl.n <= 8
+    """The library fuses the round for every global step with n <= 8."""
+    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.n <= 8
 
 
 def bytes_per_param_fused_last(wl) -> int:
     """Fused last local step + global step: per worker read x_i, the optimizer state and g and write the
-    state back (x_i is not written); read and write x and m; no replica reset."""
+    state back (x_i is not written); read and write x and m (and the global AdamW second moment); no
+    replica reset."""
     g = 2 if wl.hp.grad_dtype == W.BF16 else 4
     states = 2 if wl.hp.base == W.BASE_ADAMW else 1
-    return wl.n * (4 + 8 * states + g) + 16
+    return wl.n * (4 + 8 * states + g) + 16 + (8 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0)
 
 
 def measured_peaks():

@@ -102,7 +102,7 @@ extern "C" {
  * it), so its new replicas never go to memory, and the reset of the replicas
  * is lazy: the next round's first local step starts every worker from x
  * instead of reading n copies of it.  Applies with n <= 8 to every global
- * step but DSM_GLOBAL_ADAMW; other settings run unfused.  Reading a replica while
+ * step; more workers run unfused.  Reading a replica while
  * the reset is pending returns x; reading or writing worker state, or
  * writing gradients through dsm_fill_synthetic_grads/dsm_load_grads, while
  * the last local step is pending first runs that step unfused.  Gradients

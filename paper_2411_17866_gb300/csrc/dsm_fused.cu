@@ -17,8 +17,9 @@ namespace {
 // (tau = 1); kFusedZeroState, the base-optimizer states are zero and not read
 // (the round restarts the base optimizer and tau = 1); kFusedDropState, the
 // new states are not written (the round restarts the base optimizer).
-// kVariants: the global step is g.mode (SlowMo, signed SlowMo or Lookahead)
-// instead of Algorithm 1's.
+// kGlobal: the global step, kGlobalSign (Algorithm 1's), kGlobalRuntime
+// (g.mode: SlowMo, signed SlowMo or Lookahead, which keep x and m), or
+// kGlobalAdamW (the global AdamW step, which also keeps the second moment v).
 // A CTA walks its tiles worker by worker; each thread keeps the next
 // kFusedDepth (tile, worker) items in flight with cp.async into its own
 // shared-memory slots (x_i, m_i, v_i, g_i, and x, m with a tile's first worker).
@@ -27,14 +28,19 @@ namespace {
 // gives 0.92 / 1.00 of the copy bandwidth on GPT-2 S (AdamW, n = 4) / L
 // (SGD-momentum, n = 8), depth 3 gives 0.85 on GPT-2 M (AdamW, n = 8) where
 // depth 2 gives 0.79).
-constexpr int kFusedStreams = 6;
+constexpr int kGlobalSign = 0, kGlobalRuntime = 1, kGlobalAdamW = 2;
+// staged streams per item: x_i, m_i, v_i, g_i, x, m (and the global v for the global AdamW step)
+__host__ __device__ constexpr int fused_streams(int global) { return global == kGlobalAdamW ? 7 : 6; }
 __host__ __device__ constexpr int fused_depth(bool adamw, int nw) { return (adamw && nw > 4) ? 3 : 2; }
-__host__ __device__ constexpr size_t fused_smem(int depth) { return size_t(depth) * kFusedStreams * kThreads * sizeof(float4); }
+__host__ __device__ constexpr size_t fused_smem(int depth, int streams) {
+    return size_t(depth) * streams * kThreads * sizeof(float4);
+}
 
-template <bool kAdamW, bool kBf16, int NW, bool kVariants>
+template <bool kAdamW, bool kBf16, int NW, int kGlobal>
 __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
                                                                 GlobalScalars g, int opts) {
     constexpr int kFusedDepth = fused_depth(kAdamW, NW);
+    constexpr int kFusedStreams = fused_streams(kGlobal);
     const bool from_global = opts & kFusedFromX, zero_state = opts & kFusedZeroState,
                keep_state = !(opts & kFusedDropState);
     extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
@@ -61,6 +67,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 if (w == 0) {
                     cp_async16(slot(it, 4), p.x + gi);
                     cp_async16(slot(it, 5), p.m + gi);
+                    if (kGlobal == kGlobalAdamW) cp_async16(slot(it, 6), p.gv + gi);
                 }
             }
         }
@@ -80,7 +87,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
         const float lam_l = kAdamW ? T.lam_local : 0.f, lam_g = T.lam_global;
         const uint64_t gi = td.start + e0;
         if (vector_ok(td, e0)) {
-            float x[4], m[4], dif[NW][4];
+            float x[4], m[4], gv[4] = {0.f, 0.f, 0.f, 0.f}, dif[NW][4];
 #pragma unroll
             for (int w = 0; w < NW; ++w, ++it) {
                 cp_async_wait<kFusedDepth - 1>();  // item `it` has landed
@@ -88,6 +95,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 if (w == 0) {
                     take(it, 4, x);
                     take(it, 5, m);
+                    if (kGlobal == kGlobalAdamW) take(it, 6, gv);
                 }
                 if (from_global) {
 #pragma unroll
@@ -127,7 +135,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 issue(next_issue++);
             }
             float ru[4] = {0.f, 0.f, 0.f, 0.f};
-            if (g.sign_mode != 0) {
+            if (kGlobal == kGlobalSign && g.sign_mode != 0) {
                 const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
                 ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
             }
@@ -136,8 +144,10 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 float d[NW];
 #pragma unroll
                 for (int w = 0; w < NW; ++w) d[w] = dif[w][j];
-                if (kVariants) {
+                if (kGlobal == kGlobalRuntime) {
                     global_elem_rt<NW>(x[j], m[j], d, g, lam_g, ru[j], st);
+                } else if (kGlobal == kGlobalAdamW) {
+                    global_elem<NW, 4>(x[j], m[j], gv[j], d, NW, g, lam_g, ru[j], st);
                 } else {
                     float unused = 0.f;
                     global_elem<NW, 0>(x[j], m[j], unused, d, NW, g, lam_g, ru[j], st);
@@ -145,6 +155,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
             }
             store4(p.x + gi, x);
             store4(p.m + gi, m);
+            if (kGlobal == kGlobalAdamW) store4(p.gv + gi, gv);
         } else {
             // this thread issued no copies for the tile; keep the group count in step
 #pragma unroll
@@ -168,9 +179,14 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                     d[w] = __fsub_rn(x, xi);
                 }
                 float r = 0.f;
-                if (g.sign_mode != 0) r = philox_unit(word_of(philox_block(gj >> 2, g.philox_k0, g.philox_k1), gj & 3));
-                if (kVariants) {
+                if (kGlobal == kGlobalSign && g.sign_mode != 0)
+                    r = philox_unit(word_of(philox_block(gj >> 2, g.philox_k0, g.philox_k1), gj & 3));
+                if (kGlobal == kGlobalRuntime) {
                     global_elem_rt<NW>(x, m, d, g, lam_g, r, st);
+                } else if (kGlobal == kGlobalAdamW) {
+                    float v = p.gv[gj];
+                    global_elem<NW, 4>(x, m, v, d, NW, g, lam_g, r, st);
+                    p.gv[gj] = v;
                 } else {
                     float unused = 0.f;
                     global_elem<NW, 0>(x, m, unused, d, NW, g, lam_g, r, st);
@@ -192,38 +208,48 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
 
 using FusedKernel = void (*)(Problem, AdamScalars, SgdmScalars, GlobalScalars, int);
 
-template <bool kAdamW, bool kBf16, bool kVariants>
+template <bool kAdamW, bool kBf16, int kGlobal>
 FusedKernel fused_kernel_n(uint32_t n) {
     switch (n) {
-        case 1: return k_fused_last_global<kAdamW, kBf16, 1, kVariants>;
-        case 2: return k_fused_last_global<kAdamW, kBf16, 2, kVariants>;
-        case 3: return k_fused_last_global<kAdamW, kBf16, 3, kVariants>;
-        case 4: return k_fused_last_global<kAdamW, kBf16, 4, kVariants>;
-        case 5: return k_fused_last_global<kAdamW, kBf16, 5, kVariants>;
-        case 6: return k_fused_last_global<kAdamW, kBf16, 6, kVariants>;
-        case 7: return k_fused_last_global<kAdamW, kBf16, 7, kVariants>;
-        case 8: return k_fused_last_global<kAdamW, kBf16, 8, kVariants>;
+        case 1: return k_fused_last_global<kAdamW, kBf16, 1, kGlobal>;
+        case 2: return k_fused_last_global<kAdamW, kBf16, 2, kGlobal>;
+        case 3: return k_fused_last_global<kAdamW, kBf16, 3, kGlobal>;
+        case 4: return k_fused_last_global<kAdamW, kBf16, 4, kGlobal>;
+        case 5: return k_fused_last_global<kAdamW, kBf16, 5, kGlobal>;
+        case 6: return k_fused_last_global<kAdamW, kBf16, 6, kGlobal>;
+        case 7: return k_fused_last_global<kAdamW, kBf16, 7, kGlobal>;
+        case 8: return k_fused_last_global<kAdamW, kBf16, 8, kGlobal>;
         default: return nullptr;
     }
 }
 
-template <bool kVariants>
+template <int kGlobal>
 FusedKernel fused_kernel_v(const Problem& p, bool adamw) {
-    if (adamw) return p.grad_bf16 ? fused_kernel_n<true, true, kVariants>(p.n) : fused_kernel_n<true, false, kVariants>(p.n);
-    return p.grad_bf16 ? fused_kernel_n<false, true, kVariants>(p.n) : fused_kernel_n<false, false, kVariants>(p.n);
+    if (adamw) return p.grad_bf16 ? fused_kernel_n<true, true, kGlobal>(p.n) : fused_kernel_n<true, false, kGlobal>(p.n);
+    return p.grad_bf16 ? fused_kernel_n<false, true, kGlobal>(p.n) : fused_kernel_n<false, false, kGlobal>(p.n);
+}
+
+int fused_global_for(const Problem& p) {
+    return p.global_mode == 0 ? kGlobalSign : (p.global_mode == 4 ? kGlobalAdamW : kGlobalRuntime);
 }
 
 FusedKernel fused_kernel_for(const Problem& p, bool adamw) {
-    return p.global_mode == 0 ? fused_kernel_v<false>(p, adamw) : fused_kernel_v<true>(p, adamw);
+    switch (fused_global_for(p)) {
+        case kGlobalSign: return fused_kernel_v<kGlobalSign>(p, adamw);
+        case kGlobalAdamW: return fused_kernel_v<kGlobalAdamW>(p, adamw);
+        default: return fused_kernel_v<kGlobalRuntime>(p, adamw);
+    }
 }
 
-size_t fused_smem_for(const Problem& p, bool adamw) { return fused_smem(fused_depth(adamw, int(p.n))); }
+size_t fused_smem_for(const Problem& p, bool adamw) {
+    return fused_smem(fused_depth(adamw, int(p.n)), fused_streams(fused_global_for(p)));
+}
 
 }  // namespace
 
 bool fused_round_available(const Problem& p) {
-    // the global AdamW step keeps a third stream (v) and runs unfused
-    return p.global_mode >= 0 && p.global_mode <= 3 && p.n >= 1 && p.n <= kMaxUnrolledWorkers;
+    // every global step, up to 8 workers (the differences x - x_i of all workers stay in registers)
+    return p.global_mode >= 0 && p.global_mode <= 4 && p.n >= 1 && p.n <= kMaxUnrolledWorkers;
 }
 
 cudaError_t query_fused_shape(const Problem& p, LaunchShape* out) {

@@ -90,6 +90,10 @@ VARIANTS = [
     ("lookahead-sgdm-n8", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_LOOKAHEAD), 8, 1),
     ("global-adamw-bf16-n4", dataclasses.replace(ADAMW, grad_dtype=W.BF16, global_mode=W.GLOBAL_ADAMW), 4, 2),
     ("global-adamw-n9-generic", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_ADAMW), 9, 1),
+    ("global-adamw-sgdm-n8-t1", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_ADAMW,
+                                                     g_b1=0.8, g_b2=0.9), 8, 1),
+    ("global-adamw-f32-n1-t3", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_ADAMW, g_wd=0.0), 1, 3),
+    ("global-adamw-bf16-n6-t2", dataclasses.replace(ADAMW, grad_dtype=W.BF16, global_mode=W.GLOBAL_ADAMW), 6, 2),
     ("slowmo-n16-generic", dataclasses.replace(SGDM, sign_mode=W.SIGN, global_mode=W.GLOBAL_SLOWMO), 16, 1),
 ]
 
@@ -99,7 +103,7 @@ VARIANTS = [
 @pytest.mark.parametrize("name,hp,n,tau", VARIANTS, ids=[c[0] for c in VARIANTS])
 def test_global_variants_bitexact(layout_name, name, hp, n, tau, fused):
     """The ablations' global steps (SlowMo, signed SlowMo, Lookahead, global AdamW), three rounds,
-    in the unfused and the fused round (global AdamW and n > 8 fall back to unfused)."""
+    in the unfused and the fused round (n > 8 falls back to unfused)."""
     tensors = RAGGED if layout_name == "ragged" else MINI
     hp = dataclasses.replace(hp, flags=W.FLAG_FUSED_ROUND if fused else 0)
     run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
