@@ -650,10 +650,11 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     g.philox_k1 = static_cast<uint32_t>(h->t & 0xFFFFFFFFull);
     cudaStream_t s = S(stream);
     cudaError_t err;
+    uint32_t grid = 0;  // CTAs of the global-step launch (the statistics reduction needs it)
     if (h->last_pending) {  // fused round: last local step + global step, reset left pending
         const int opts = (h->replicas_stale ? kFusedFromX : 0) | (h->states_zero ? kFusedZeroState : 0) |
                          (h->reset_local ? kFusedDropState : 0);
-        err = launch_fused_last_global(h->prob, h->shape, h->pending_a, h->pending_sa, g, opts, s);
+        err = launch_fused_last_global(h->prob, h->shape, h->pending_a, h->pending_sa, g, opts, s, &grid);
         if (err != cudaSuccess) return cuda_fail(err, "launch fused last local step and global step");
         h->last_pending = false;
         h->replicas_stale = true;
@@ -661,10 +662,10 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     } else {
         int rc = materialize_replicas(h, s);
         if (rc != DSM_OK) return rc;
-        err = launch_global(h->prob, h->shape, g, s);
+        err = launch_global(h->prob, h->shape, g, s, &grid);
         if (err != cudaSuccess) return cuda_fail(err, "launch global step");
     }
-    err = launch_stats(h->prob, s);
+    err = launch_stats(h->prob, grid, s);
     if (err != cudaSuccess) return cuda_fail(err, "launch statistics");
     h->t += 1;
     h->k = 0;

@@ -329,15 +329,6 @@ __device__ __forceinline__ void reduce_stats(const ThreadStats& st, StatPartial*
     __syncthreads();  // the shared arrays are reused by the next reduction
 }
 
-__device__ __forceinline__ void zero_partial(StatPartial* out) {
-    if (threadIdx.x == 0) {
-        StatPartial p;
-        p.delta_sq = 0.0; p.drift = 0.0;
-        p.zero_sign = p.flips = p.unanimous = p.clamped = 0;
-        *out = p;
-    }
-}
-
 // Per-thread asynchronous global -> shared copies (cp.async): the copy holds
 // no register while in flight, and a thread waits only for its own groups.
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {

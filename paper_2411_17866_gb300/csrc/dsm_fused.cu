@@ -197,10 +197,8 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
         }
         const uint32_t next = ti + gridDim.x;
         if (next >= p.num_tiles || p.tiles[next].tensor != td.tensor) {  // uniform across the CTA
-            reduce_stats(st, p.partials + ti);
+            reduce_stats(st, p.partials + ti);  // a CTA's last tile of this tensor (as in K4)
             st = ThreadStats();
-        } else {
-            zero_partial(p.partials + ti);
         }
     }
     cp_async_wait<0>();  // the groups issued past the last tile are empty; nothing is left in flight
@@ -263,9 +261,11 @@ cudaError_t query_fused_shape(const Problem& p, LaunchShape* out) {
 }
 
 cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
-                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s) {
+                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s,
+                                     uint32_t* grid_used) {
     if (!fused_round_available(p)) return cudaErrorInvalidValue;
     const int grid = clamp_grid(ls.grid_fused, p.num_tiles);
+    *grid_used = static_cast<uint32_t>(grid);
     if (grid == 0) return cudaSuccess;
     fused_kernel_for(p, p.opt_v != nullptr)<<<grid, kThreads, fused_smem_for(p, p.opt_v != nullptr), s>>>(
         p, a, sa, g, opts);

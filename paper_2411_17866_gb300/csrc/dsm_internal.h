@@ -75,7 +75,7 @@ struct Problem {
     float* opt_v;          // [n][d_stride] (AdamW only)
     void* grad;            // [n][d_stride], fp32 or bf16
     int grad_bf16;
-    StatPartial* partials; // [num_tiles]
+    StatPartial* partials; // [num_tiles]; only each CTA's last tile of a tensor is written
     TensorStats* stats;    // [num_tensors]
 };
 
@@ -137,10 +137,14 @@ constexpr int kFusedZeroState = 2;  // the base-optimizer states are zero: none 
 constexpr int kFusedDropState = 4;  // the new base-optimizer states are not written (the round resets them)
 bool fused_round_available(const Problem& p);
 cudaError_t query_fused_shape(const Problem& p, LaunchShape* out);  // sets grid_fused (out->sms must be set)
+// The global-step launchers write per-tile statistics partials and set *grid to the number of CTAs
+// they launched; launch_stats reduces those partials per tensor and needs that grid.
 cudaError_t launch_fused_last_global(const Problem& p, const LaunchShape& ls, const AdamScalars& a,
-                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s);
-cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s);
-cudaError_t launch_stats(const Problem& p, cudaStream_t s);
+                                     const SgdmScalars& sa, const GlobalScalars& g, int opts, cudaStream_t s,
+                                     uint32_t* grid);
+cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s,
+                          uint32_t* grid);
+cudaError_t launch_stats(const Problem& p, uint32_t producer_grid, cudaStream_t s);
 
 // Sets the calling thread's message returned by dsm_last_error() (dsm_api.cpp).
 void set_last_error_message(const char* msg);

@@ -406,8 +406,10 @@ __device__ __forceinline__ void global_vec_generic(const Problem& p, const Globa
 // NW == 0: any n, one element at a time.
 // Statistics: a CTA keeps per-thread sums while its successive tiles belong
 // to one tensor and reduces them only when the tensor changes (or at its last
-// tile), writing the segment's partial at the segment's last tile and zeros
-// at its other tiles; the per-tensor sum over tiles is then unchanged.
+// tile), writing the segment's partial at the segment's last tile.  With a
+// grid of G CTAs, tile t is a CTA's last tile of its tensor exactly when
+// t + G lies beyond the tensor, so the partials of a tensor are its last
+// min(G, tiles) tiles, which K5 sums.
 template <int NW, int MODE>
 __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g) {
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
@@ -478,19 +480,21 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
         if (next >= p.num_tiles || nt.tensor != td.tensor) {  // uniform across the CTA
             reduce_stats(st, p.partials + ti);
             st = ThreadStats();
-        } else {
-            zero_partial(p.partials + ti);
         }
     }
 }
 
-// K5: per-tensor statistics from the tile partials, in a fixed order.
-__global__ void __launch_bounds__(kThreads) k_stats(Problem p) {
+// K5: per-tensor statistics from the tile partials, in a fixed order: a
+// tensor's partials are its last min(G, tiles) tiles for a producing grid of
+// G CTAs (see K4).
+__global__ void __launch_bounds__(kThreads) k_stats(Problem p, uint32_t producer_grid) {
     const uint32_t T = blockIdx.x;
     const TensorDesc td = p.tensors[T];
     double a = 0.0, b = 0.0;
     unsigned long long c0 = 0, c1 = 0, c2 = 0, c3 = 0;
-    for (uint32_t t = td.tile_begin + threadIdx.x; t < td.tile_end; t += blockDim.x) {
+    const uint32_t first =
+        td.tile_end - td.tile_begin > producer_grid ? td.tile_end - producer_grid : td.tile_begin;
+    for (uint32_t t = first + threadIdx.x; t < td.tile_end; t += blockDim.x) {
         const StatPartial q = p.partials[t];
         a += q.delta_sq; b += q.drift;
         c0 += q.zero_sign; c1 += q.flips; c2 += q.unanimous; c3 += q.clamped;
@@ -638,16 +642,18 @@ cudaError_t launch_local_sgdm(const Problem& p, const LaunchShape& ls, const Sgd
     return cudaGetLastError();
 }
 
-cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s) {
+cudaError_t launch_global(const Problem& p, const LaunchShape& ls, const GlobalScalars& g, cudaStream_t s,
+                          uint32_t* grid_used) {
     const int grid = clamp_grid(ls.grid_global, p.num_tiles);
+    *grid_used = static_cast<uint32_t>(grid);
     if (grid == 0) return cudaSuccess;
     global_kernel_for(p.n, p.global_mode)<<<grid, kThreads, 0, s>>>(p, g);
     return cudaGetLastError();
 }
 
-cudaError_t launch_stats(const Problem& p, cudaStream_t s) {
+cudaError_t launch_stats(const Problem& p, uint32_t producer_grid, cudaStream_t s) {
     if (p.num_tensors == 0) return cudaSuccess;
-    k_stats<<<p.num_tensors, kThreads, 0, s>>>(p);
+    k_stats<<<p.num_tensors, kThreads, 0, s>>>(p, producer_grid);
     return cudaGetLastError();
 }
 

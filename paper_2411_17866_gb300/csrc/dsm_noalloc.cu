@@ -229,8 +229,9 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     g.sign_mode = hp->sign_mode;
     g.philox_k0 = static_cast<uint32_t>(hp->seed & 0xFFFFFFFFull);
     g.philox_k1 = static_cast<uint32_t>(round & 0xFFFFFFFFull);
-    if ((err = launch_global(p, ls, g, s)) != cudaSuccess) return na_cuda(err, "launch global step");
-    if ((err = launch_stats(p, s)) != cudaSuccess) return na_cuda(err, "launch statistics");
+    uint32_t grid = 0;
+    if ((err = launch_global(p, ls, g, s, &grid)) != cudaSuccess) return na_cuda(err, "launch global step");
+    if ((err = launch_stats(p, grid, s)) != cudaSuccess) return na_cuda(err, "launch statistics");
     if (stats) {
         err = cudaMemcpyAsync(stats, p.stats, sizeof(TensorStats) * layout->count,
                               stats_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, s);
