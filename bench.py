@@ -41,7 +41,7 @@ METRIC = "params/s per global round (τ local + sign-momentum step); % HBM roofl
 UNIT = "params/s"
 CPU_SAMPLE_ELEMS = 1 << 22
 # the sources of the local-step kernels (their arithmetic lives in the shared device header)
-KERNELS_SRC = [os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", f) for f in ("dsm_device.cuh", "dsm_kernels.cu")]
+KERNELS_SRC = [os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", f) for f in ("dsm_device.cuh", "dsm_local.cu")]
 
 
 def kernels_source_hash() -> str:

@@ -1,6 +1,6 @@
 """Builds libdsm.so, the C-ABI library, in-tree for sm_103a (GB300).
 
-The two translation units compile in parallel, then link into a shared
+The translation units compile in parallel, then link into a shared
 library next to this file.  No CMake; nvcc and the host compiler only.
 """
 from __future__ import annotations
@@ -24,7 +24,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # and square root are nvcc's defaults and stay on.
 NVCC_FLAGS = ["-O3", "-lineinfo", "--fmad=false", "-std=c++17", "-Xcompiler", "-fPIC",
               "-Xcompiler", "-ffp-contract=off", "-I" + INCLUDE, "-I" + CSRC]
-SOURCES = ["dsm_kernels.cu", "dsm_fused.cu", "dsm_api.cpp", "dsm_noalloc.cu"]
+SOURCES = ["dsm_kernels.cu", "dsm_local.cu", "dsm_fused.cu", "dsm_api.cpp", "dsm_noalloc.cu"]
 
 
 def nvcc() -> str:

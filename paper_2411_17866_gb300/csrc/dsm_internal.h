@@ -119,8 +119,9 @@ struct LaunchShape {
     int grid_fused = 0, grid_adamw_from_x = 0, grid_sgdm_from_x = 0;
 };
 
-// Launchers (dsm_kernels.cu).  Each returns the cudaError_t of its launch.
+// Launchers (dsm_kernels.cu, dsm_local.cu, dsm_fused.cu).  Each returns the cudaError_t of its launch.
 cudaError_t query_launch_shape(const Problem& p, LaunchShape* out);
+cudaError_t query_local_shape(const Problem& p, LaunchShape* out);  // the local steps' grids (dsm_local.cu)
 cudaError_t launch_init(const Problem& p, const LaunchShape& ls, uint64_t seed_key_init, int from_hash,
                         cudaStream_t s);
 cudaError_t launch_grad_fill(const Problem& p, const LaunchShape& ls, const GradKeys& k, cudaStream_t s);
