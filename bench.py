@@ -153,14 +153,21 @@ def bytes_per_elem_local(wl) -> int:
     return 4 * 4 + g          # read x, buf, g; write x, buf
 
 
-def bytes_per_param_global(wl) -> int:
-    # read x, m (and the global AdamW second moment) and n replicas; write them all
-    return 8 * (wl.n + 2 + (1 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0))
+def bytes_per_param_global(wl, lazy_reset=False) -> int:
+    # read x, m (and the global AdamW second moment) and n replicas; write them all (the replicas
+    # only when the reset is not deferred)
+    return 8 * (wl.n + 2 + (1 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0)) - (4 * wl.n if lazy_reset else 0)
 
 
 def fused_round_active(wl) -> bool:
-    """The library fuses the round for every global step with n <= 8."""
+    """The library runs the last local step inside the global step with n <= 8 workers."""
     return bool(wl.hp.flags & W.FLAG_FUSED_ROUND) and wl.n <= 8
+
+
+def lazy_reset_active(wl) -> bool:
+    """With the fused-round flag the replicas' reset is deferred for any n: the next round's first
+    local step starts every worker from x."""
+    return bool(wl.hp.flags & W.FLAG_FUSED_ROUND)
 
 
 def bytes_per_param_fused_last(wl) -> int:
@@ -349,6 +356,7 @@ def main():
     tau = wl.tau
 
     fused = fused_round_active(wl)
+    lazy = lazy_reset_active(wl)
     local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
     local_bytes_from_x = wl.n * wl.d * (bytes_per_elem_local(wl) - 4) + wl.d * 4
 
@@ -369,8 +377,8 @@ def main():
                 a.record(stream)
                 run.local_step(stream)
                 b.record(stream)
-                # fused round: the first local step starts every worker from x (read once per tile)
-                nbytes = local_bytes_from_x if (fused and k == 0 and t > 0) else local_bytes
+                # deferred reset: the first local step starts every worker from x (read once per tile)
+                nbytes = local_bytes_from_x if (lazy and k == 0 and t > 0) else local_bytes
                 local_events.append((a, b, nbytes))
             else:
                 run.local_step(stream)
@@ -451,7 +459,7 @@ def main():
 
     peak, peak_kind = measured_peaks()
     # fused round: the last local step runs inside the global-step launch
-    global_bytes = wl.d * (bytes_per_param_global(wl) if not fused else bytes_per_param_fused_last(wl))
+    global_bytes = wl.d * (bytes_per_param_global(wl, lazy) if not fused else bytes_per_param_fused_last(wl))
     avg_local_s = statistics.mean(local_ms) / 1e3
     grad_bytes = wl.n * wl.d * (2 if wl.hp.grad_dtype == W.BF16 else 4)
     achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
@@ -472,7 +480,8 @@ def main():
                         "achieved_gbs": global_bytes / avg_global_s / 1e9,
                         "frac": global_bytes / avg_global_s / 1e9 / peak,
                         "note": ("last local step fused with the global step, + statistics reduction"
-                                 if fused else "fused global step + statistics reduction") +
+                                 if fused else "fused global step + statistics reduction" +
+                                 (" (replica reset deferred)" if lazy else "")) +
                                 ", CUDA events around both"},
         "grad_fill": {"avg_ms": statistics.mean(fill_ms), "bytes_written_per_launch": grad_bytes,
                       "write_gbs": grad_bytes / (statistics.mean(fill_ms) / 1e3) / 1e9,

@@ -101,8 +101,10 @@ extern "C" {
  * runs inside dsm_global_step (dsm_local_step for k = tau-1 only records
  * it), so its new replicas never go to memory, and the reset of the replicas
  * is lazy: the next round's first local step starts every worker from x
- * instead of reading n copies of it.  Applies with n <= 8 to every global
- * step; more workers run unfused.  Reading a replica while
+ * instead of reading n copies of it.  Applies to every global step; with
+ * more than 8 workers only the reset is deferred (the last local step runs
+ * on its own: the differences of all workers no longer fit in registers).
+ * Reading a replica while
  * the reset is pending returns x; reading or writing worker state, or
  * writing gradients through dsm_fill_synthetic_grads/dsm_load_grads, while
  * the last local step is pending first runs that step unfused.  Gradients

@@ -189,6 +189,7 @@ struct dsm_handle {
     double gb2_pow = 1.0;
     // fused round (DSM_FLAG_FUSED_ROUND)
     bool fused = false;           // flag set and a fused kernel exists for this problem
+    bool lazy_reset = false;      // flag set: the replicas' reset is deferred (fused kernel or not)
     bool replicas_stale = false;  // the replicas' reset to x is pending
     bool last_pending = false;    // the round's last local step waits for the global step
     // DSM_FLAG_RESET_LOCAL_STATE
@@ -466,6 +467,7 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     };
     if ((err = query_launch_shape(p, &h->shape)) != cudaSuccess) return bail(err, "occupancy query");
     h->fused = (hp->flags & DSM_FLAG_FUSED_ROUND) && fused_round_available(p);
+    h->lazy_reset = (hp->flags & DSM_FLAG_FUSED_ROUND) != 0;
     // The tables are copied from the handle's own vectors, which outlive the copies.
     if ((err = cudaMemcpyAsync(A + al.off_tensors, h->tensors.data(), h->tensors.size() * sizeof(TensorDesc),
                                cudaMemcpyHostToDevice, s)) != cudaSuccess)
@@ -662,8 +664,10 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     } else {
         int rc = materialize_replicas(h, s);
         if (rc != DSM_OK) return rc;
+        g.skip_reset = h->lazy_reset ? 1 : 0;  // more than 8 workers: only the reset is deferred
         err = launch_global(h->prob, h->shape, g, s, &grid);
         if (err != cudaSuccess) return cuda_fail(err, "launch global step");
+        if (h->lazy_reset) h->replicas_stale = true;
     }
     err = launch_stats(h->prob, grid, s);
     if (err != cudaSuccess) return cuda_fail(err, "launch statistics");

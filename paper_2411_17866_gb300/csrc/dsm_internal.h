@@ -104,6 +104,7 @@ struct GlobalScalars {
     int sign_mode;
     int mode;              // DSM_GLOBAL_*: read by the fused round's kernel for the ablation variants
     uint32_t philox_k0, philox_k1;
+    int skip_reset;        // K4: leave the replicas' reset to x pending (the next local step starts from x)
 };
 
 // SplitMix64 keys of one synthetic-gradient fill.

@@ -186,7 +186,8 @@ __device__ __forceinline__ void global_elem_generic(const Problem& p, const Glob
     p.x[gi] = x;
     p.m[gi] = m;
     if (MODE == 4) p.gv[gi] = v;
-    for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = x;
+    if (!g.skip_reset)
+        for (uint32_t i = 0; i < p.n; ++i) p.X[i * p.d_stride + gi] = x;
 }
 
 // Global step on a thread's 4 aligned elements for any number of workers:
@@ -254,7 +255,7 @@ __device__ __forceinline__ void global_vec_generic(const Problem& p, const Globa
                     dr[j] = __fadd_rn(dr[j], __fmul_rn(ei, ei));
                     unan[j] = unan[j] && (sgn(di) == sD[j]);
                 }
-                store4(p.X + (i0 + c) * p.d_stride + gi, xn);
+                if (!g.skip_reset) store4(p.X + (i0 + c) * p.d_stride + gi, xn);
             }
         }
     }
@@ -269,7 +270,7 @@ __device__ __forceinline__ void global_vec_generic(const Problem& p, const Globa
 }
 
 // K4: the fused global step (average over the replicas, sign-momentum update,
-// momentum update, reset of every replica) with statistics.
+// momentum update, reset of every replica unless g.skip_reset) with statistics.
 // NW > 0: exactly NW replicas, held in registers and double-buffered.
 // NW == 0: any n, one element at a time.
 // Statistics: a CTA keeps per-thread sums while its successive tiles belong
@@ -337,8 +338,10 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
             store4(p.x + gi, cx);
             store4(p.m + gi, cm);
             if (MODE == 4) store4(p.gv + gi, cv);
+            if (!g.skip_reset) {
 #pragma unroll
-            for (int i = 0; i < W; ++i) store4(p.X + i * p.d_stride + gi, cx);
+                for (int i = 0; i < W; ++i) store4(p.X + i * p.d_stride + gi, cx);
+            }
         } else if (NW == 0 && vector_ok(td, e0)) {
             global_vec_generic<MODE>(p, g, lam, td.start + e0, st);
         } else {

@@ -160,7 +160,7 @@ cudaError_t query_local_shape(const Problem& p, LaunchShape* out) {
     constexpr int kSgdmCtasPerSm = 4;
     out->grid_sgdm = std::min(p.grad_bf16 ? grid_for(k_local_sgdm<true, false, false>, sms)
                                           : grid_for(k_local_sgdm<false, false, false>, sms), kSgdmCtasPerSm * sms);
-    if (fused_round_available(p)) {  // the from-x variants run only in the fused round
+    {  // the from-x variants (first local step after a lazy reset)
         out->grid_adamw_from_x = std::min(p.grad_bf16 ? grid_for(k_local_adamw<true, true, false>, sms)
                                                       : grid_for(k_local_adamw<false, true, false>, sms),
                                           kAdamwCtasPerSm * sms);

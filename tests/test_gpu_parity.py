@@ -123,7 +123,8 @@ FUSED = [
     ("sgdm-rsignpm-n3-t2", dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, grad_dtype=W.BF16), 3, 2),
     ("adamw-n1-t1", ADAMW, 1, 1),
     ("adamw-n5-t2", ADAMW, 5, 2),
-    ("adamw-n9-unfused", ADAMW, 9, 2),
+    ("adamw-n9-deferred-reset", ADAMW, 9, 2),
+    ("sgdm-rsign-n16-deferred-reset", SGDM, 16, 1),
     ("slowmo-unfused", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO), 4, 2),
 ]
 
@@ -131,7 +132,8 @@ FUSED = [
 @pytest.mark.parametrize("layout_name", ["ragged", "mini"])
 @pytest.mark.parametrize("name,hp,n,tau", FUSED, ids=[c[0] for c in FUSED])
 def test_fused_round_bitexact(layout_name, name, hp, n, tau):
-    """The fused round (last local step inside the global step, lazy reset) gives the same state."""
+    """The fused round (last local step inside the global step, lazy reset; above 8 workers the lazy
+    reset alone) gives the same state."""
     tensors = RAGGED if layout_name == "ragged" else MINI
     hp = dataclasses.replace(hp, flags=W.FLAG_FUSED_ROUND)
     run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
@@ -555,6 +557,7 @@ HOST_GRADS = [
     ("adamw-bf16-n8-t2", dataclasses.replace(ADAMW, grad_dtype=W.BF16), 8, 2),
     ("sgdm-n4-t1-fused", dataclasses.replace(SGDM, flags=W.FLAG_FUSED_ROUND), 4, 1),
     ("adamw-n9-generic-t2", ADAMW, 9, 2),
+    ("adamw-n9-t2-deferred-reset", dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND), 9, 2),
     ("reset-adamw-n4-t3-fused", dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND | W.FLAG_RESET_LOCAL_STATE), 4, 3),
 ]
 
