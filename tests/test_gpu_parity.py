@@ -624,3 +624,24 @@ def test_host_gradient_steps_mix_with_device_fills():
     with pytest.raises(ValueError):
         run.local_step_host_grads(torch.zeros((n, d + 1)))
     run.close()
+
+
+SMALL = (W.Tensor("s9", 9, W.KIND_WEIGHT, 1e-2), W.Tensor("s1000", 1000, W.KIND_WEIGHT, 1e-3),
+         W.Tensor("s1", 1, W.KIND_LN_W, 1e-3), W.Tensor("s8", 8, W.KIND_BIAS, 1e-3),
+         W.Tensor("s1024", 1024, W.KIND_WEIGHT, 1e-3), W.Tensor("s1025", 1025, W.KIND_LN_B, 1e-4))
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+@pytest.mark.parametrize("name,hp,n", [("adamw-n2", ADAMW, 2), ("sgdm-rsign-n5", SGDM, 5)], ids=["adamw-n2", "sgdm-rsign-n5"])
+def test_small_tensors_tau4(name, hp, n, fused):
+    """Tensors of 9, 1000, 1, 8, 1024 and 1025 elements (sub-tile, exactly one tile, one past a tile),
+    four local steps per round, three rounds."""
+    hp = dataclasses.replace(hp, flags=W.FLAG_FUSED_ROUND if fused else 0)
+    run = dsm.DistributedSignMomentum(SMALL, n, 4, hp)
+    ora = O.OracleRun(SMALL, n, 4, hp, with_stats=True)
+    for _ in range(3):
+        stats = run.synthetic_round(with_stats=True)
+        ora.run_round()
+        compare_state(run, ora)
+        compare_stats(stats, ora.last_stats, n)
+    run.close()
