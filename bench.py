@@ -273,8 +273,55 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(rows), "power_w_max": pmax, "gpu": self.gpu}
 
 
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _oracle_slice_worker(tensors, n, tau, hp, start, count, warmup, steps, barrier, out):
+    """One process of the all-cores oracle run: rounds over elements [start, start + count)."""
+    import numpy as np
+
+    from oracle import dsm_oracle as O
+    ora = O.OracleRun(tensors, n, tau, hp, elems=np.arange(start, start + count, dtype=np.int64))
+    for _ in range(warmup):
+        ora.run_round()
+    for step in range(steps):
+        barrier.wait()
+        t0 = time.time()
+        ora.run_round()
+        out.put((step, t0, time.time()))
+
+
+def parallel_oracle(wl, per_worker, workers, steps=1, warmup=0):
+    """The CPU oracle, as it stands, in `workers` processes over consecutive element slices of
+    `per_worker` elements (every step is elementwise, so slices are independent).  Processes start
+    with spawn (the parent holds a CUDA context); a barrier starts each step in all of them, and a
+    step's time is the first start to the last finish.  Returns (elements, step wall times)."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    per_worker = max(1, min(per_worker, wl.d // workers))
+    barrier, out = ctx.Barrier(workers), ctx.Queue()
+    procs = [ctx.Process(target=_oracle_slice_worker,
+                         args=(wl.tensors, wl.n, wl.tau, wl.hp, i * per_worker, per_worker, warmup, steps, barrier,
+                               out)) for i in range(workers)]
+    for p in procs:
+        p.start()
+    marks = [out.get() for _ in range(workers * steps)]
+    for p in procs:
+        p.join()
+    walls = []
+    for step in range(steps):
+        t = [(a, b) for st, a, b in marks if st == step]
+        walls.append(max(b for _, b in t) - min(a for a, _ in t))
+    return per_worker * workers, walls
+
+
 def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, rounds=1):
-    """The CPU oracle, as it stands, on one round over a contiguous sample of the workload."""
+    """The CPU oracle, as it stands: one round over a contiguous sample of the workload on every host
+    core (one process per core, one slice each), and the same on one core."""
     import numpy as np
 
     from oracle import dsm_oracle as O
@@ -284,10 +331,15 @@ def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, rounds=1):
     for _ in range(rounds):
         ora.run_round()
     dt = time.perf_counter() - t0
-    return {"value": count * rounds / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+    one = {"value": count * rounds / dt, "cores": 1,
+           "sample": f"{rounds} round(s) over elements [0, {count}), one thread; {dt:.2f} s"}
+    cores = host_cores()
+    total, walls = parallel_oracle(wl, count, cores, steps=rounds)
+    return {"value": total * rounds / sum(walls), "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"{rounds} round(s) (tau={wl.tau} local steps x n={wl.n} workers + global step) over "
-                      f"elements [0, {count}) of the {wl.d}-parameter layout, numpy fp32, one thread; "
-                      f"{dt:.2f} s"}
+                      f"elements [0, {total}) of the {wl.d}-parameter layout, numpy fp32, {cores} processes "
+                      f"of {total // cores} consecutive elements each; {sum(walls):.2f} s",
+            "one_core": one}
 
 
 def run_reference(args):
@@ -295,29 +347,23 @@ def run_reference(args):
     if rank != 0:
         return 0
     wl = select_workload(args)
-    import numpy as np
-
-    from oracle import dsm_oracle as O
     # each step one round over a contiguous sample, sized so that the whole run stays near a minute of
     # CPU time whatever --steps and --warmup are (about 2^20 elements per step at the defaults)
     per_step = (1 << 20) * (20 + 3) // max(1, args.steps + args.warmup)
     per_step = per_step * 48 // (wl.n * wl.tau)          # the defaults' n*tau is 48
     count = int(min(max(per_step, 1 << 14), 1 << 22, wl.d))
-    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64))
-    for _ in range(args.warmup):
-        ora.run_round()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        ora.run_round()
-    dt = time.perf_counter() - t0
-    value = count * args.steps / dt
+    cores = host_cores()
+    total, walls = parallel_oracle(wl, count, cores, steps=args.steps, warmup=args.warmup)
+    dt = sum(walls)
+    value = total * args.steps / dt
     sample = (f"each step: one round (tau={wl.tau} x n={wl.n} local steps + global step) over elements "
-              f"[0, {count}) of the {wl.d}-parameter layout; numpy fp32 oracle, one thread")
+              f"[0, {total}) of the {wl.d}-parameter layout; numpy fp32 oracle in {cores} processes of "
+              f"{total // cores} consecutive elements each")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic", "config": workload_config(wl, args.gpus),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
