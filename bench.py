@@ -72,6 +72,8 @@ def parse():
     ap.add_argument("--global-mode", default=None, choices=sorted(GLOBAL_MODES))
     # fused round (default): the last local step inside the global step, lazy replica reset
     ap.add_argument("--no-fused", dest="fused", action="store_false")
+    # the variant in which every round restarts each worker's base optimizer from zero state
+    ap.add_argument("--reset-local-state", action="store_true")
     return ap.parse_args()
 
 
@@ -101,6 +103,10 @@ def select_workload(args):
         changes["hp"] = dataclasses.replace(hp, flags=hp.flags | W.FLAG_FUSED_ROUND)
     else:
         notes.append("unfused round")
+    if args.reset_local_state:   # a variant of the method: every round restarts the base optimizer
+        hp = changes.get("hp", wl.hp)
+        changes["hp"] = dataclasses.replace(hp, flags=hp.flags | W.FLAG_RESET_LOCAL_STATE)
+        notes.append("base optimizer restarted every round")
     if args.max_params:
         keep, total = [], 0
         for t in wl.tensors:
@@ -111,7 +117,8 @@ def select_workload(args):
         changes["tensors"] = tuple(keep)
         notes.append(f"reduced to the first {len(keep)} tensors ({total} params)")
     if changes:
-        changes["name"] = wl.name + " [" + ", ".join(notes) + "]"
+        if notes:
+            changes["name"] = wl.name + " [" + ", ".join(notes) + "]"
         wl = dataclasses.replace(wl, **changes)
     return wl
 
@@ -145,12 +152,20 @@ def whole_job_value(d_per_rank: int, world: int, rounds: int, seconds: float) ->
     return world * d_per_rank * rounds / seconds
 
 
-def bytes_per_elem_local(wl) -> int:
-    """Algorithmic bytes of one local step per worker-element: every state read and written once."""
+def bytes_per_elem_local(wl, zero_state=False) -> int:
+    """Algorithmic bytes of one local step per worker-element: every state read and written once
+    (zero_state: the base optimizer restarts, its state is written but not read)."""
     g = 2 if wl.hp.grad_dtype == W.BF16 else 4
-    if wl.hp.base == W.BASE_ADAMW:
-        return 6 * 4 + g      # read x, m, v, g; write x, m, v
-    return 4 * 4 + g          # read x, buf, g; write x, buf
+    states = 2 if wl.hp.base == W.BASE_ADAMW else 1
+    # read x, the states and g; write x and the states
+    return 4 + 4 * states * (1 if zero_state else 2) + g + 4
+
+
+def local_step_bytes(wl, from_x=False, zero_state=False) -> int:
+    """Algorithmic bytes of one local-step launch (from_x: every worker starts from the global x,
+    read once per tile)."""
+    b = bytes_per_elem_local(wl, zero_state)
+    return wl.n * wl.d * (b - 4) + wl.d * 4 if from_x else wl.n * wl.d * b
 
 
 def bytes_per_param_global(wl, lazy_reset=False) -> int:
@@ -170,13 +185,16 @@ def lazy_reset_active(wl) -> bool:
     return bool(wl.hp.flags & W.FLAG_FUSED_ROUND)
 
 
-def bytes_per_param_fused_last(wl) -> int:
-    """Fused last local step + global step: per worker read x_i, the optimizer state and g and write the
-    state back (x_i is not written); read and write x and m (and the global AdamW second moment); no
-    replica reset."""
+def bytes_per_param_fused_last(wl, from_x=False, zero_state=False) -> int:
+    """Fused last local step + global step: per worker read x_i (unless every worker starts from x),
+    the optimizer state (unless it restarts from zero) and g, and write the state back (not when the
+    round restarts the base optimizer; x_i is never written); read and write x and m (and the global
+    AdamW second moment); no replica reset."""
     g = 2 if wl.hp.grad_dtype == W.BF16 else 4
     states = 2 if wl.hp.base == W.BASE_ADAMW else 1
-    return wl.n * (4 + 8 * states + g) + 16 + (8 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0)
+    reset = bool(wl.hp.flags & W.FLAG_RESET_LOCAL_STATE)
+    per_worker = (0 if from_x else 4) + g + (0 if zero_state else 4 * states) + (0 if reset else 4 * states)
+    return wl.n * per_worker + 16 + (8 if wl.hp.global_mode == W.GLOBAL_ADAMW else 0)
 
 
 def measured_peaks():
@@ -403,8 +421,8 @@ def main():
 
     fused = fused_round_active(wl)
     lazy = lazy_reset_active(wl)
-    local_bytes = wl.n * wl.d * bytes_per_elem_local(wl)
-    local_bytes_from_x = wl.n * wl.d * (bytes_per_elem_local(wl) - 4) + wl.d * 4
+    reset = bool(wl.hp.flags & W.FLAG_RESET_LOCAL_STATE)
+    local_bytes = local_step_bytes(wl)
 
     def round_(t, local_events=None, global_events=None, fill_events=None):
         for k in range(tau):
@@ -423,8 +441,9 @@ def main():
                 a.record(stream)
                 run.local_step(stream)
                 b.record(stream)
-                # deferred reset: the first local step starts every worker from x (read once per tile)
-                nbytes = local_bytes_from_x if (lazy and k == 0 and t > 0) else local_bytes
+                # deferred reset: the first local step starts every worker from x (read once per tile);
+                # restarted base optimizer: the first local step reads no state
+                nbytes = local_step_bytes(wl, from_x=lazy and k == 0 and t > 0, zero_state=reset and k == 0 and t > 0)
                 local_events.append((a, b, nbytes))
             else:
                 run.local_step(stream)
@@ -434,7 +453,12 @@ def main():
             a.record(stream)
             run.global_step(stream)
             b.record(stream)
-            global_events.append((a, b))
+            if fused:   # with tau = 1 the fused launch is also the round's first local step
+                first = tau == 1 and t > 0
+                gbytes = wl.d * bytes_per_param_fused_last(wl, from_x=first, zero_state=reset and first)
+            else:
+                gbytes = wl.d * bytes_per_param_global(wl, lazy)
+            global_events.append((a, b, gbytes))
         else:
             run.global_step(stream)
 
@@ -465,7 +489,8 @@ def main():
     elapsed = max_over_ranks(start.elapsed_time(end) / 1e3, world)
     local_ms = [a.elapsed_time(b) for a, b, _ in local_ev]
     local_launch_bytes = [nb for _, _, nb in local_ev]
-    global_ms = [a.elapsed_time(b) for a, b in global_ev]
+    global_ms = [a.elapsed_time(b) for a, b, _ in global_ev]
+    global_launch_bytes = [nb for _, _, nb in global_ev]
     fill_ms = [a.elapsed_time(b) for a, b in fill_ev]
 
     # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device
@@ -505,13 +530,20 @@ def main():
 
     peak, peak_kind = measured_peaks()
     # fused round: the last local step runs inside the global-step launch
-    global_bytes = wl.d * (bytes_per_param_global(wl, lazy) if not fused else bytes_per_param_fused_last(wl))
-    avg_local_s = statistics.mean(local_ms) / 1e3
+    global_bytes = statistics.mean(global_launch_bytes)
     grad_bytes = wl.n * wl.d * (2 if wl.hp.grad_dtype == W.BF16 else 4)
-    achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
-    kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
-    traffic = committed_traffic(f"{kname}:{args.workload}")
+    global_gbs = sum(global_launch_bytes) / (sum(global_ms) / 1e3) / 1e9
     avg_global_s = statistics.mean(global_ms) / 1e3
+    if local_ms:   # the dominant kernel: the local step
+        avg_local_s = statistics.mean(local_ms) / 1e3
+        achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
+        kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
+        # the traffic record holds for the workload as configured by default (a full local-step launch)
+        default = wl.name == W.WORKLOADS[args.workload].name
+        traffic = committed_traffic(f"{kname}:{args.workload}") if default else None
+    else:          # tau = 1 in the fused round: the only launch is the fused last step + global step
+        avg_local_s, achieved, kname, traffic = avg_global_s, global_gbs, "fused_last_global", None
+        local_bytes = global_bytes
     value = whole_job_value(wl.d, world, args.steps, elapsed)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -523,8 +555,7 @@ def main():
                      "traffic": traffic, "algorithmic_bytes_per_launch": local_bytes,
                      "avg_launch_ms": avg_local_s * 1e3},
         "global_step": {"bytes_per_launch": global_bytes, "avg_ms": avg_global_s * 1e3,
-                        "achieved_gbs": global_bytes / avg_global_s / 1e9,
-                        "frac": global_bytes / avg_global_s / 1e9 / peak,
+                        "achieved_gbs": global_gbs, "frac": global_gbs / peak,
                         "note": ("last local step fused with the global step, + statistics reduction"
                                  if fused else "fused global step + statistics reduction" +
                                  (" (replica reset deferred)" if lazy else "")) +
