@@ -645,3 +645,34 @@ def test_small_tensors_tau4(name, hp, n, fused):
         compare_state(run, ora)
         compare_stats(stats, ora.last_stats, n)
     run.close()
+
+
+def test_two_handles_on_two_streams_are_independent():
+    """Two handles (different base optimizers, sign modes and fused settings) whose rounds are issued
+    alternately on two streams: each equals its own oracle bit for bit."""
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    hp_a = dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND, seed=21)
+    hp_b = dataclasses.replace(SGDM, seed=22)
+    a = dsm.DistributedSignMomentum(RAGGED, 3, 2, hp_a)
+    b = dsm.DistributedSignMomentum(MINI, 5, 3, hp_b)
+    oa = O.OracleRun(RAGGED, 3, 2, hp_a)
+    ob = O.OracleRun(MINI, 5, 3, hp_b)
+    torch.cuda.synchronize()
+    for t in range(2):
+        for k in range(3):
+            if k < 2:
+                a.fill_synthetic_grads(t * 2 + k, s1)
+                a.local_step(s1)
+                oa.local_step()
+            b.fill_synthetic_grads(t * 3 + k, s2)
+            b.local_step(s2)
+            ob.local_step()
+        a.global_step(s1)
+        b.global_step(s2)
+        oa.global_step()
+        ob.global_step()
+    torch.cuda.synchronize()
+    compare_state(a, oa)
+    compare_state(b, ob)
+    a.close()
+    b.close()
