@@ -246,6 +246,18 @@ int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream);
  * worker >= n. */
 int dsm_grad_ptr(dsm_handle* h, uint32_t worker, void** dev_ptr);
 
+/* Device address of worker `worker`'s current model x^{(i)} (d fp32 values,
+ * the caller must not write through it), the point at which Eq. (base-sgd)
+ * evaluates that worker's stochastic gradient: a framework runs its forward
+ * and backward pass over views of this memory, then writes the gradients
+ * through dsm_grad_ptr.  While the replicas' reset is pending (fused round)
+ * the address is that of x itself; if the round's last local step is
+ * pending, the call first runs it on stream.  The address and its contents
+ * stay valid until the next call that changes the state (a local or global
+ * step, a write of worker state).  DSM_EINVAL for NULL arguments, DSM_ERANGE
+ * for worker >= n, DSM_ECUDA if the pending step fails to launch. */
+int dsm_replica_ptr(dsm_handle* h, uint32_t worker, dsm_stream_t stream, const float** dev_ptr);
+
 /* Copy all workers' gradients (the grad f_i of Eq. (base-sgd)) from src, a
  * dense [n][d] array of the gradient type in host (src_is_device = 0;
  * pinned memory makes it asynchronous) or device memory, into the gradient

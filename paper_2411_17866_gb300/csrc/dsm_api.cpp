@@ -521,6 +521,17 @@ int dsm_grad_ptr(dsm_handle* h, uint32_t worker, void** dev_ptr) {
     return DSM_OK;
 }
 
+int dsm_replica_ptr(dsm_handle* h, uint32_t worker, dsm_stream_t stream, const float** dev_ptr) {
+    if (!h || !dev_ptr) return fail(DSM_EINVAL, "NULL argument");
+    if (worker >= h->n) return fail(DSM_ERANGE, "worker %u >= n = %u", worker, h->n);
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    int rc = materialize_pending(h, S(stream));
+    if (rc != DSM_OK) return rc;
+    *dev_ptr = h->replicas_stale ? h->prob.x : h->prob.X + uint64_t(worker) * h->al.d_stride;
+    return DSM_OK;
+}
+
 int dsm_load_grads(dsm_handle* h, const void* src, int src_is_device, dsm_stream_t stream) {
     if (!h || !src) return fail(DSM_EINVAL, "NULL argument");
     DeviceGuard guard(h->device);

@@ -75,6 +75,7 @@ _PROTOS = {
     "dsm_set_gamma": (c_int, [c_void_p, c_float]),
     "dsm_fill_synthetic_grads": (c_int, [c_void_p, c_uint64, c_void_p]),
     "dsm_grad_ptr": (c_int, [c_void_p, c_uint32, POINTER(c_void_p)]),
+    "dsm_replica_ptr": (c_int, [c_void_p, c_uint32, c_void_p, POINTER(c_void_p)]),
     "dsm_load_grads": (c_int, [c_void_p, c_void_p, c_int, c_void_p]),
     "dsm_local_step": (c_int, [c_void_p, c_void_p]),
     "dsm_local_step_host_grads": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -185,6 +186,12 @@ def dsm_fill_synthetic_grads(h, step: int, stream=None) -> None:
 def dsm_grad_ptr(h, worker: int) -> int:
     p = c_void_p()
     _check(load_library().dsm_grad_ptr(h, worker, byref(p)), "dsm_grad_ptr")
+    return p.value
+
+
+def dsm_replica_ptr(h, worker: int, stream=None) -> int:
+    p = c_void_p()
+    _check(load_library().dsm_replica_ptr(h, worker, _stream(stream), byref(p)), "dsm_replica_ptr")
     return p.value
 
 
@@ -322,6 +329,28 @@ class DistributedSignMomentum:
 
     def local_step(self, stream=None):
         dsm_local_step(self.h, stream)
+
+    def _arena_view(self, ptr: int, count: int, dtype):
+        """A tensor aliasing `count` elements of the arena at device address `ptr`."""
+        import torch
+        esize = torch.tensor([], dtype=dtype).element_size()
+        off = ptr - self.arena.data_ptr()
+        if off < 0 or off + count * esize > self.nbytes:
+            raise DsmError(DSM_ERANGE, "_arena_view", "address outside the arena")
+        return self.arena[off:off + count * esize].view(dtype)
+
+    def replica_view(self, worker, stream=None):
+        """Worker `worker`'s current model x^(i) as a read-only-by-contract float32 CUDA tensor of d
+        elements (aliasing the arena; valid until the next step or state write)."""
+        import torch
+        return self._arena_view(dsm_replica_ptr(self.h, worker, stream), self.d, torch.float32)
+
+    def grad_view(self, worker):
+        """Worker `worker`'s gradient buffer as a CUDA tensor of d elements of the gradient type
+        (aliasing the arena), for a caller that writes its own gradients."""
+        import torch
+        dt = torch.bfloat16 if self.hp.grad_dtype == BF16 else torch.float32
+        return self._arena_view(dsm_grad_ptr(self.h, worker), self.d, dt)
 
     def local_step_host_grads(self, src, stream=None, copy_stream=None):
         """One local step on gradients in host memory (``src``: [n, d] CPU tensor of the gradient type,
