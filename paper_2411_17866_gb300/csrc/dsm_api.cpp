@@ -290,6 +290,20 @@ cudaError_t launch_local(dsm_handle* h, const AdamScalars& a, const SgdmScalars&
     return err;
 }
 
+// Records a local step as done: deferred to the global step (fused round, last step) or launched.
+void count_local_step(dsm_handle* h, bool deferred, const AdamScalars& a, const SgdmScalars& sa, double nb1,
+                      double nb2) {
+    if (deferred) {
+        h->pending_a = a;
+        h->pending_sa = sa;
+        h->last_pending = true;
+    }
+    h->b1_pow = nb1;
+    h->b2_pow = nb2;
+    h->j += 1;
+    h->k += 1;
+}
+
 // Chunks of whole tiles for dsm_local_step_host_grads: about kChunkBytes of gradients (all
 // workers) each, at most kMaxChunks, and their events (created on first use).
 constexpr uint64_t kChunkBytes = 64ull << 20;
@@ -562,18 +576,12 @@ int dsm_local_step(dsm_handle* h, dsm_stream_t stream) {
     SgdmScalars sa;
     double nb1, nb2;
     next_local_scalars(h, &a, &sa, &nb1, &nb2);
-    if (h->fused && h->k + 1 == h->tau) {  // the last step runs inside dsm_global_step
-        h->pending_a = a;
-        h->pending_sa = sa;
-        h->last_pending = true;
-    } else {
+    const bool defer = h->fused && h->k + 1 == h->tau;  // the last step runs inside dsm_global_step
+    if (!defer) {
         cudaError_t err = launch_local(h, a, sa, S(stream));
         if (err != cudaSuccess) return cuda_fail(err, "launch local step");  // the handle is unchanged
     }
-    h->b1_pow = nb1;
-    h->b2_pow = nb2;
-    h->j += 1;
-    h->k += 1;
+    count_local_step(h, defer, a, sa, nb1, nb2);
     return DSM_OK;
 }
 
@@ -617,17 +625,8 @@ int dsm_local_step_host_grads(dsm_handle* h, const void* src, dsm_stream_t strea
             if (err != cudaSuccess) return cuda_fail(err, "launch the local step on a chunk");
         }
     }
-    if (defer) {
-        h->pending_a = a;
-        h->pending_sa = sa;
-        h->last_pending = true;
-    } else {
-        h->replicas_stale = h->states_zero = false;
-    }
-    h->b1_pow = nb1;
-    h->b2_pow = nb2;
-    h->j += 1;
-    h->k += 1;
+    if (!defer) h->replicas_stale = h->states_zero = false;
+    count_local_step(h, defer, a, sa, nb1, nb2);
     return DSM_OK;
 }
 
