@@ -676,3 +676,41 @@ def test_two_handles_on_two_streams_are_independent():
     compare_state(b, ob)
     a.close()
     b.close()
+
+
+@pytest.mark.parametrize("name,hp", [("adamw", ADAMW), ("sgdm-rsign", SGDM)], ids=["adamw", "sgdm-rsign"])
+def test_non_finite_gradients_propagate_like_the_oracle(name, hp):
+    """Gradients holding +inf, -inf and NaN at a few elements: the GPU state equals the oracle's, with
+    NaN compared as NaN (the payload bits of a NaN are not fixed by IEEE 754) and every finite value
+    bit for bit; the sign of a NaN argument is 0 on both sides."""
+    tensors, n, tau = MINI, 3, 2
+    d = sum(t.numel for t in tensors)
+    run = dsm.DistributedSignMomentum(tensors, n, tau, hp)
+    ora = O.OracleRun(tensors, n, tau, hp)
+    rng = np.random.default_rng(5)
+    for t in range(2):
+        for k in range(tau):
+            g = (rng.standard_normal((n, d)) * 1e-3).astype(np.float32)
+            g[0, 10], g[1, 20], g[2, 30 + t] = np.inf, -np.inf, np.nan
+            g[1, 40 + k] = np.float32(3e38)
+            run.load_grads(torch.from_numpy(g).cuda())
+            run.local_step()
+            with np.errstate(all="ignore"):
+                ora.local_step([g[i] for i in range(n)])
+        run.global_step()
+        with np.errstate(all="ignore"):
+            ora.global_step()
+
+    def same(got, want, what):
+        got = np.asarray(got)
+        nan_g, nan_w = np.isnan(got), np.isnan(want)
+        assert np.array_equal(nan_g, nan_w), f"{what}: NaN positions differ"
+        assert np.array_equal(got[~nan_g].view(np.uint32), np.asarray(want, np.float32)[~nan_w].view(np.uint32)), what
+    same(run.read(dsm.BUF_X).numpy(), ora.x, "x")
+    same(run.read(dsm.BUF_M).numpy(), ora.m, "m")
+    for i in range(n):
+        same(run.read(dsm.BUF_REPLICA, i).numpy(), ora.X[i], f"replica {i}")
+        same(run.read(dsm.BUF_OPT_M, i).numpy(), ora.opt_m[i], f"opt_m {i}")
+        if ora.opt_v is not None:
+            same(run.read(dsm.BUF_OPT_V, i).numpy(), ora.opt_v[i], f"opt_v {i}")
+    run.close()
