@@ -59,7 +59,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--workload", default=W.BENCH_WORKLOAD, choices=sorted(W.WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -505,16 +505,22 @@ def main():
             run.read(dsm.BUF_GRAD, i, out=host_g[i], stream=stream)
         host_x = torch.empty(wl.d, dtype=torch.float32).pin_memory()
         copy_stream = torch.cuda.Stream(dev)
-        torch.cuda.synchronize()
-        if world > 1:
-            dist.barrier()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
+
+        def e2e_round():
             for k in range(tau):
                 # the copy of each chunk of gradients overlaps the update of the previous chunk
                 run.local_step_host_grads(host_g, stream, copy_stream)
             run.global_step(stream)
             run.read(dsm.BUF_X, out=host_x, stream=stream)   # synchronises the stream
+
+        e2e_round()   # one untimed round: first use of the pinned buffers and of the chunk events
+        t += 1
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_round()
             t += 1
         e2e_dt = max_over_ranks(time.perf_counter() - t0, world)
         e2e = {"value": whole_job_value(wl.d, world, args.e2e_steps, e2e_dt), "unit": UNIT,

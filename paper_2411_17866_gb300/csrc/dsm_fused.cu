@@ -22,31 +22,49 @@ namespace {
 // kGlobalAdamW (the global AdamW step, which also keeps the second moment v).
 // A CTA walks its tiles worker by worker; each thread keeps the next
 // kFusedDepth (tile, worker) items in flight with cp.async into its own
-// shared-memory slots (x_i, m_i, v_i, g_i, and x, m with a tile's first worker).
+// shared-memory slots: x_i, m_i (v_i) and g_i per item, and x, m with a tile's
+// first worker into a slot pair kept per tile parity.
 // Items in flight per thread: 2, or 3 for AdamW with more than 4 workers,
 // whose registers already limit the resident CTAs (measured on GB300: depth 2
 // gives 0.92 / 1.00 of the copy bandwidth on GPT-2 S (AdamW, n = 4) / L
 // (SGD-momentum, n = 8), depth 3 gives 0.85 on GPT-2 M (AdamW, n = 8) where
-// depth 2 gives 0.79).
+// depth 2 gives 0.79).  Staging x and m once per tile instead of in every
+// item's slots (59 instead of 72 KB per CTA for GPT-2 M) raised GPT-2 M to
+// 0.87; four items in flight in the same 72 KB gave 0.86.
 constexpr int kGlobalSign = 0, kGlobalRuntime = 1, kGlobalAdamW = 2;
-// staged streams per item: x_i, m_i, v_i, g_i, x, m (and the global v for the global AdamW step)
-__host__ __device__ constexpr int fused_streams(int global) { return global == kGlobalAdamW ? 7 : 6; }
 __host__ __device__ constexpr int fused_depth(bool adamw, int nw) { return (adamw && nw > 4) ? 3 : 2; }
-__host__ __device__ constexpr size_t fused_smem(int depth, int streams) {
-    return size_t(depth) * streams * kThreads * sizeof(float4);
+// Staging per thread: for every item in flight the worker's x_i, m_i (and v_i
+// for AdamW) in 16-byte slots and its gradient in an 8- or 16-byte slot; for
+// each of two tiles (by parity) x and m (and the global v) of the tile.
+__host__ __device__ constexpr int fused_states(bool adamw) { return adamw ? 3 : 2; }
+__host__ __device__ constexpr int fused_globals(int global) { return global == kGlobalAdamW ? 3 : 2; }
+__host__ __device__ constexpr size_t fused_smem(bool adamw, bool bf16, int nw, int global) {
+    return (size_t(fused_depth(adamw, nw)) * (fused_states(adamw) * 16 + (bf16 ? 8 : 16)) +
+            2 * fused_globals(global) * 16) * kThreads;
 }
 
 template <bool kAdamW, bool kBf16, int NW, int kGlobal>
 __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamScalars a, SgdmScalars sa,
                                                                 GlobalScalars g, int opts) {
     constexpr int kFusedDepth = fused_depth(kAdamW, NW);
-    constexpr int kFusedStreams = fused_streams(kGlobal);
+    constexpr int kStates = fused_states(kAdamW), kGlobals = fused_globals(kGlobal);
+    constexpr int kGradBytes = kBf16 ? 8 : 16;
+    static_assert(kFusedDepth <= 2 * NW, "a tile's x and m slots are reused two tiles later");
     const bool from_global = opts & kFusedFromX, zero_state = opts & kFusedZeroState,
                keep_state = !(opts & kFusedDropState);
-    extern __shared__ float4 fsm[];  // [kFusedDepth][kFusedStreams][kThreads]
+    // [kFusedDepth][kStates][kThreads] float4 | [kFusedDepth][kThreads] gradients | [2][kGlobals][kThreads] float4
+    extern __shared__ float4 fsm[];
+    char* const grad_base = reinterpret_cast<char*>(fsm + size_t(kFusedDepth) * kStates * kThreads);
+    float4* const glob_base = reinterpret_cast<float4*>(grad_base + size_t(kFusedDepth) * kThreads * kGradBytes);
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
-    auto slot = [&](int it, int stream) -> float4* {
-        return fsm + (size_t(it % kFusedDepth) * kFusedStreams + stream) * kThreads + threadIdx.x;
+    auto state_slot = [&](uint32_t it, int s) -> float4* {
+        return fsm + (size_t(it % kFusedDepth) * kStates + s) * kThreads + threadIdx.x;
+    };
+    auto grad_slot = [&](uint32_t it) -> void* {
+        return grad_base + (size_t(it % kFusedDepth) * kThreads + threadIdx.x) * kGradBytes;
+    };
+    auto glob_slot = [&](uint32_t q, int s) -> float4* {
+        return glob_base + (size_t(q & 1) * kGlobals + s) * kThreads + threadIdx.x;
     };
     // Issue item `it` (tile number it / NW of this CTA, worker it % NW); always commits one group.
     auto issue = [&](uint32_t it) {
@@ -57,24 +75,24 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
             if (vector_ok(t, e0)) {
                 const uint64_t gi = t.start + e0;
                 const uint64_t o = w * p.d_stride + gi;
-                if (!from_global) cp_async16(slot(it, 0), p.X + o);
+                if (!from_global) cp_async16(state_slot(it, 0), p.X + o);
                 if (!zero_state) {
-                    cp_async16(slot(it, 1), p.opt_m + o);
-                    if (kAdamW) cp_async16(slot(it, 2), p.opt_v + o);
+                    cp_async16(state_slot(it, 1), p.opt_m + o);
+                    if (kAdamW) cp_async16(state_slot(it, 2), p.opt_v + o);
                 }
-                if (kBf16) cp_async8(slot(it, 3), reinterpret_cast<const __nv_bfloat16*>(p.grad) + o);
-                else cp_async16(slot(it, 3), reinterpret_cast<const float*>(p.grad) + o);
+                if (kBf16) cp_async8(grad_slot(it), reinterpret_cast<const __nv_bfloat16*>(p.grad) + o);
+                else cp_async16(grad_slot(it), reinterpret_cast<const float*>(p.grad) + o);
                 if (w == 0) {
-                    cp_async16(slot(it, 4), p.x + gi);
-                    cp_async16(slot(it, 5), p.m + gi);
-                    if (kGlobal == kGlobalAdamW) cp_async16(slot(it, 6), p.gv + gi);
+                    cp_async16(glob_slot(q, 0), p.x + gi);
+                    cp_async16(glob_slot(q, 1), p.m + gi);
+                    if (kGlobal == kGlobalAdamW) cp_async16(glob_slot(q, 2), p.gv + gi);
                 }
             }
         }
         cp_async_commit();
     };
-    auto take = [&](int it, int stream, float (&v)[4]) {
-        const float4 t = *slot(it, stream);
+    auto take = [&](const float4* src, float (&v)[4]) {
+        const float4 t = *src;
         v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
     };
     uint32_t next_issue = 0;
@@ -93,31 +111,32 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 cp_async_wait<kFusedDepth - 1>();  // item `it` has landed
                 float xi[4], mi[4], vi[4], gr[4];
                 if (w == 0) {
-                    take(it, 4, x);
-                    take(it, 5, m);
-                    if (kGlobal == kGlobalAdamW) take(it, 6, gv);
+                    const uint32_t q = it / NW;
+                    take(glob_slot(q, 0), x);
+                    take(glob_slot(q, 1), m);
+                    if (kGlobal == kGlobalAdamW) take(glob_slot(q, 2), gv);
                 }
                 if (from_global) {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) xi[j] = x[j];
                 } else {
-                    take(it, 0, xi);
+                    take(state_slot(it, 0), xi);
                 }
                 if (zero_state) {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) mi[j] = vi[j] = 0.f;
                 } else {
-                    take(it, 1, mi);
-                    if (kAdamW) take(it, 2, vi);
+                    take(state_slot(it, 1), mi);
+                    if (kAdamW) take(state_slot(it, 2), vi);
                 }
                 if (kBf16) {
-                    const uint2 raw = *reinterpret_cast<const uint2*>(slot(it, 3));
+                    const uint2 raw = *reinterpret_cast<const uint2*>(grad_slot(it));
                     gr[0] = __uint_as_float(raw.x << 16);
                     gr[1] = __uint_as_float(raw.x & 0xFFFF0000u);
                     gr[2] = __uint_as_float(raw.y << 16);
                     gr[3] = __uint_as_float(raw.y & 0xFFFF0000u);
                 } else {
-                    take(it, 3, gr);
+                    take(reinterpret_cast<const float4*>(grad_slot(it)), gr);
                 }
                 const uint64_t o = w * p.d_stride + gi;
 #pragma unroll
@@ -240,7 +259,7 @@ FusedKernel fused_kernel_for(const Problem& p, bool adamw) {
 }
 
 size_t fused_smem_for(const Problem& p, bool adamw) {
-    return fused_smem(fused_depth(adamw, int(p.n)), fused_streams(fused_global_for(p)));
+    return fused_smem(adamw, p.grad_bf16 != 0, int(p.n), fused_global_for(p));
 }
 
 }  // namespace
