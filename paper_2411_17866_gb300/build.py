@@ -24,7 +24,8 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # and square root are nvcc's defaults and stay on.
 NVCC_FLAGS = ["-O3", "-lineinfo", "--fmad=false", "-std=c++17", "-Xcompiler", "-fPIC",
               "-Xcompiler", "-ffp-contract=off", "-I" + INCLUDE, "-I" + CSRC]
-SOURCES = ["dsm_kernels.cu", "dsm_local.cu", "dsm_fused.cu", "dsm_api.cpp", "dsm_noalloc.cu"]
+SOURCES = ["dsm_kernels.cu", "dsm_local.cu", "dsm_fused.cu", "dsm_fused_sign.cu", "dsm_fused_variants.cu",
+           "dsm_fused_adamw.cu", "dsm_api.cpp", "dsm_noalloc.cu"]
 
 
 def nvcc() -> str:
