@@ -166,3 +166,27 @@ def test_host_memory_arena_is_refused(lib):
     assert rc in (dsm.DSM_ECUDA, dsm.DSM_EALIGN)
     msg = dsm.last_error()
     assert ("device memory" in msg) if rc == dsm.DSM_EALIGN else ("cudaPointerGetAttributes" in msg)
+
+
+def test_header_constants_match_the_python_side():
+    """Every integer constant the header defines has the same value in the binding and, where the
+    workload definitions use it, in workloads.py."""
+    src = open(HEADER).read()
+    defs = {m.group(1): int(m.group(2).rstrip("u"), 0)
+            for m in re.finditer(r"#define\s+(DSM_[A-Z0-9_]+)\s+\(?(-?(?:0x[0-9A-Fa-f]+|\d+)u?)\)?", src)}
+    assert len(defs) >= 30
+    checked = 0
+    for name, value in defs.items():
+        if name.startswith("DSM_NOALLOC_"):
+            continue
+        short = name[len("DSM_"):]
+        if name in ("DSM_OK", "DSM_EINVAL", "DSM_ENOMEM", "DSM_EALIGN", "DSM_ESTATE", "DSM_ECUDA", "DSM_ERANGE"):
+            assert getattr(dsm, name) == value, name
+            checked += 1
+            continue
+        assert hasattr(dsm, short), f"{name} has no counterpart in the binding"
+        assert getattr(dsm, short) == value, name
+        checked += 1
+        if hasattr(W, short):
+            assert getattr(W, short) == value, name
+    assert checked == len([n for n in defs if not n.startswith("DSM_NOALLOC_")])
