@@ -21,6 +21,9 @@ What it computes (arXiv 2411.17866):
 * The global-step variants of the ablations (Sec. 5): SlowMo (Appendix A,
   Algorithm "SlowMo"), signed SlowMo and Lookahead (Sec. 5, ablation
   studies), and the global AdamW step (Appendix, Algorithm "global AdamW").
+* Both readings of what Algorithm 1 leaves open about the base optimizer's
+  state at a synchronisation: kept across rounds (the default), or restarted
+  from zero every round (FLAG_RESET_LOCAL_STATE).
 
 Precision.  The paper fixes no precision.  Every function is generic in the
 float dtype: ``np.float32`` is the canonical mode whose expression trees the
