@@ -97,11 +97,14 @@ __device__ __forceinline__ void load4_bf16(const __nv_bfloat16* p, float (&v)[4]
     v[3] = __uint_as_float(raw.y & 0xFFFF0000u);
 }
 
+// fp32 -> bf16 rounds to nearest even, two values per conversion (the first in the low half).
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 __device__ __forceinline__ void store4_bf16(__nv_bfloat16* p, const float (&v)[4]) {
-    uint32_t h[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) h[i] = __bfloat16_as_ushort(__float2bfloat16_rn(v[i]));
-    __stcs(reinterpret_cast<uint2*>(p), make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16)));
+    __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3])));
 }
 
 template <bool kBf16>
