@@ -10,7 +10,9 @@ arena tensor and a handle and exposes the round as Python methods.
 """
 from __future__ import annotations
 
+import collections
 import ctypes
+import math
 import os
 from ctypes import POINTER, byref, c_char_p, c_float, c_int, c_int32, c_size_t, c_uint32, c_uint64, c_void_p
 
@@ -145,6 +147,9 @@ def make_layout(tensors):
     lay = dsm_layout(ctypes.cast(arr, POINTER(dsm_tensor)), len(tensors))
     lay._keep = arr
     return lay
+
+
+LayoutEntry = collections.namedtuple("LayoutEntry", "numel grad_scale kind wd")
 
 
 def make_hparams(hp) -> dsm_hparams:
@@ -294,6 +299,8 @@ class DistributedSignMomentum:
     elements (host or device).
     """
 
+    shapes = None   # the tensors' shapes, for a problem built by from_tensors
+
     def __init__(self, tensors, n: int, tau: int, hp, device="cuda", x0=None, stream=None):
         import torch
         self.layout = make_layout(tensors)
@@ -316,6 +323,37 @@ class DistributedSignMomentum:
         info = dsm_get_info(self.h)
         self.d, self.d_stride = int(info.d), int(info.d_stride)
         self.num_tensors = int(info.num_tensors)
+
+    @classmethod
+    def from_tensors(cls, params, n: int, tau: int, hp, device="cuda", decay=None, stream=None):
+        """A problem over the given tensors (e.g. a torch module's parameters, in order): one layout
+        entry per tensor (kind weight for tensors of two or more dimensions, bias otherwise; decoupled
+        weight decay on every tensor unless ``decay``, one bool per tensor, says otherwise), and the
+        initial model x0 = their current values, concatenated.  ``unflatten`` splits a flat buffer
+        back into tensors of these shapes."""
+        import torch
+        params = [p.detach() for p in params]
+        decay = [True] * len(params) if decay is None else list(decay)
+        if len(decay) != len(params):
+            raise ValueError("decay needs one entry per tensor")
+        layout = [LayoutEntry(int(p.numel()), 0.0, KIND_WEIGHT if p.dim() >= 2 else KIND_BIAS, int(bool(wd)))
+                  for p, wd in zip(params, decay)]
+        x0 = torch.cat([p.reshape(-1).to(torch.float32) for p in params]).to(device)
+        obj = cls(layout, n, tau, hp, device=device, x0=x0, stream=stream)
+        obj.shapes = [tuple(p.shape) for p in params]
+        return obj
+
+    def unflatten(self, flat):
+        """Views of a flat d-element tensor (a replica, x, a gradient buffer) shaped like the tensors
+        given to from_tensors."""
+        if self.shapes is None:
+            raise ValueError("unflatten needs a problem built by from_tensors")
+        out, off = [], 0
+        for shape in self.shapes:
+            k = math.prod(shape)
+            out.append(flat[off:off + k].view(shape))
+            off += k
+        return out
 
     # Algorithm 1, one call per step
     def set_gamma(self, gamma):

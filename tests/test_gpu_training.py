@@ -108,3 +108,52 @@ def test_replica_view_follows_the_lazy_reset():
         dsm.dsm_replica_ptr(run.h, 2)
     assert e.value.code == dsm.DSM_ERANGE
     run.close()
+
+
+def test_training_a_module_built_from_its_parameters():
+    """DistributedSignMomentum.from_tensors over a torch module's parameters (its current values are x0),
+    unflatten for the per-worker parameter views: 20 rounds, bit-exact against the oracle started from
+    the same x0, and the loss falls."""
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.manual_seed(3)
+    model = torch.nn.Sequential(torch.nn.Linear(IN, HID), torch.nn.ReLU(), torch.nn.Linear(HID, OUT))
+    params = list(model.parameters())
+    hp = W.HParams(lr=1e-2, wd=0.0, g_eta=1.0, g_b1=0.95, g_b2=0.98, g_wd=0.0, flags=W.FLAG_FUSED_ROUND)
+    run = dsm.DistributedSignMomentum.from_tensors(params, N, TAU, hp)
+    assert run.shapes == [tuple(p.shape) for p in params]
+    x0 = torch.cat([p.detach().reshape(-1) for p in params]).numpy()
+    tensors = tuple(W.Tensor(f"p{i}", p.numel(), W.KIND_WEIGHT if p.dim() > 1 else W.KIND_BIAS, 0.0)
+                    for i, p in enumerate(params))
+    ora = O.OracleRun(tensors, N, TAU, hp, x0=x0)
+
+    def forward(p, X):
+        return torch.nn.functional.linear(torch.relu(torch.nn.functional.linear(X, p[0], p[1])), p[2], p[3])
+
+    centers = torch.randn(OUT, IN, generator=torch.Generator().manual_seed(0))
+    X_eval, y_eval = _batch(centers, list(range(OUT)), torch.Generator().manual_seed(99))
+    X_eval, y_eval = X_eval.cuda(), y_eval.cuda()
+    gens = [torch.Generator().manual_seed(40 + i) for i in range(N)]
+
+    def eval_loss():
+        return float(torch.nn.functional.cross_entropy(forward(run.unflatten(run.read(dsm.BUF_X).cuda()), X_eval),
+                                                       y_eval))
+
+    loss0 = eval_loss()
+    for t in range(20):
+        for k in range(TAU):
+            grads = []
+            for i in range(N):
+                p = [q.detach().requires_grad_() for q in run.unflatten(run.replica_view(i))]
+                X, y = _batch(centers, WORKER_CLASSES[i], gens[i])
+                gr = torch.autograd.grad(torch.nn.functional.cross_entropy(forward(p, X.cuda()), y.cuda()), p)
+                flat = torch.cat([q.reshape(-1) for q in gr])
+                run.grad_view(i).copy_(flat)
+                grads.append(flat.cpu().numpy())
+            run.local_step()
+            ora.local_step(grads)
+        run.global_step()
+        ora.global_step()
+    torch.cuda.synchronize()
+    compare_state(run, ora)
+    assert eval_loss() < 0.8 * loss0
+    run.close()
