@@ -84,3 +84,11 @@ def test_client_rounds_match_the_oracle(client, kind):
         assert [int(v) for v in got[4:8]] == [want["zero_sign"], want["flips"], want["unanimous"], want["clamped"]]
         for v, key in ((float(got[2]), "delta_sq"), (float(got[3]), "drift")):
             assert abs(v - want[key]) <= stats_rtol(4) * abs(want[key])
+
+
+def test_header_is_cxx11():
+    if shutil.which("g++") is None:
+        pytest.skip("no C++ compiler")
+    r = subprocess.run(["g++", "-std=c++11", "-Wall", "-Wextra", "-Werror", "-pedantic", "-fsyntax-only", "-x", "c++",
+                        os.path.join(ROOT, "include", "dsm.h")], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
