@@ -1,17 +1,18 @@
 // CUDA kernels (sm_103a) for one global round of distributed sign momentum
 // with local steps (arXiv 2411.17866, Algorithm 1): initialisation, the
 // synthetic gradients (K1), the global step (K4) and its statistics (K5).
-// The local steps are in dsm_local.cu, the fused round in dsm_fused.cu.
+// The local steps are in dsm_local.cu, the fused round in dsm_fused.cuh.
 //
 // Every kernel is a persistent, grid-stride loop over work items: tiles of
 // at most kTile = 1024 elements that lie inside one tensor (for the local
 // steps, a tile of one worker).  A CTA of 256 threads takes one item at a
 // time; each thread owns 4 consecutive elements and moves them with one
 // 16-byte load or store per fp32 stream (8 bytes per bf16 stream), so every
-// warp instruction covers 512 contiguous bytes.  The local and global steps
-// double-buffer in registers: a thread issues the loads of its next item
-// before it computes the current one, so the HBM requests of one item are in
-// flight during the arithmetic of the previous one.  The work is streaming and
+// warp instruction covers 512 contiguous bytes.  (K1 instead runs 64-thread
+// CTAs whose threads own four such groups of a tile.)  The local and global
+// steps double-buffer in registers: a thread issues the loads of its next
+// item before it computes the current one, so the HBM requests of one item
+// are in flight during the arithmetic of the previous one.  The work is streaming and
 // elementwise, bound by HBM bandwidth; nothing is a contraction, and no tensor
 // core is used.
 //
