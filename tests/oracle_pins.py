@@ -40,7 +40,7 @@ def pin_worked_example(o, dt=np.float32):
                    g_eta=float(Fraction(hpj["eta"])), g_wd=float(Fraction(hpj["lambda"])))
     tensors = W.flat_layout(8, 1.0)
     x0 = _frac_array(ex["x0"], np.float32)
-    run = o.OracleRun(tensors, hpj["n"], hpj["tau"], hp, x0=x0, dtype=dt)
+    run = o.OracleRun(tensors, hpj["n"], hpj["tau"], hp, x0=x0, dtype=dt, with_stats=True)
     for t, exp in enumerate(ex["rounds"]):
         grads = [[_frac_array(gi, np.float32) for gi in gk] for gk in ex["grads"]["values"][t]]
         run.run_round(grads)
@@ -51,6 +51,42 @@ def pin_worked_example(o, dt=np.float32):
             assert np.array_equal(np.asarray(got, dtype=dt), want), (t, key, got, want)
         for Xi in run.X:
             assert np.array_equal(Xi, run.x)
+        _check_stats(run.last_stats[0], exp["stats"], ("round", t))
+
+
+def _check_stats(got, want, where):
+    """Statistics against hand-computed values: dyadic sums exactly, counts exactly."""
+    for key in ("delta_sq", "drift"):
+        assert got[key] == float(Fraction(want[key])), (where, key, got[key], want[key])
+    for key in ("zero_sign", "flips", "unanimous", "clamped"):
+        assert got[key] == want[key], (where, key, got[key], want[key])
+
+
+def pin_stats_example(o):
+    """A hand-built global step (d = 8, n = 3, chosen uniforms r) whose statistics separate every count
+    from a plausible mistake: unanimity over every worker (not any, and not skipping zero differences),
+    flips of sign(u) against sign(Delta) (not of the applied randomized sign), zeros of the applied sign,
+    clamping strictly above B; and the randomized signs' comparison r < p (strict)."""
+    ex = _load("stats_example_d8.json")
+    hpj = ex["hparams"]
+    dt = np.float32
+    x = _frac_array(ex["x"], dt)
+    m = _frac_array(ex["m"], dt)
+    X = [x - _frac_array(di, dt) for di in ex["diffs"]["values"]]
+    r = _frac_array(ex["r"], dt)
+    lam = np.full(8, float(Fraction(hpj["lambda"])), dtype=dt)
+    B = float(Fraction(hpj["B"]))
+    gamma, b1, b2, eta = (float(Fraction(hpj[k])) for k in ("gamma", "beta1", "beta2", "eta"))
+    for mode_name, mode in (("sign", 0), ("rand_sign_2", 1), ("rand_sign_1", 2)):
+        want = ex["modes"][mode_name]
+        x_new, m_new, inter = o.global_step(x, m, X, gamma, b1, b2, eta, lam, mode, B, r, np.dtype(dt))
+        for key, got in (("delta", inter["delta"]), ("u", inter["u"]), ("m_new", m_new)):
+            assert np.array_equal(got, _frac_array(ex[key], dt)), (mode_name, key, got)
+        sg = _frac_array(want["sign"], dt)
+        assert np.array_equal(inter["sg"], sg), (mode_name, inter["sg"], sg)
+        assert np.array_equal(x_new, (-float(Fraction(eta)) * float(Fraction(gamma)) * sg).astype(dt)), mode_name
+        st = o.round_stats(inter, np.zeros(8, dtype=np.int64), 1, mode, B)
+        _check_stats(st[0], want["stats"], mode_name)
 
 
 # ---------------------------------------------------------------------------
@@ -590,7 +626,7 @@ def pin_cosine_schedule(o):
     assert all(a >= b for a, b in zip(vals, vals[1:]))
 
 
-PINS = [pin_worked_example, pin_splitmix64, pin_philox, pin_philox_uniform_mapping, pin_bf16,
+PINS = [pin_worked_example, pin_stats_example, pin_splitmix64, pin_philox, pin_philox_uniform_mapping, pin_bf16,
         pin_uniform24, pin_hash_fields, pin_synthetic_grad, pin_adamw_vs_torch, pin_adamw_constant_grad,
         pin_adamw_first_step_fp32, pin_sgdm_vs_torch, pin_sgd_plain_exact, pin_sgdm_constant_grad,
         pin_lion, pin_signsgd_momentum, pin_identical_workers, pin_tau1_pseudo_gradient,

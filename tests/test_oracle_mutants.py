@@ -74,6 +74,29 @@ MUTANTS = [
      [P.pin_synthetic_grad]),
     ("stats_drift_uncentred", "drift_e += (dd - delta) ** 2", "drift_e += dd ** 2",
      [P.pin_stats]),
+    ("stats_unanimous_any_worker",
+     "    unanimous = np.ones(delta.shape, dtype=bool)\n    for dd_, dd in zip(inter[\"diffs\"], diffs):\n"
+     "        unanimous &= sign(dd_) == sd",
+     "    unanimous = np.zeros(delta.shape, dtype=bool)\n    for dd_, dd in zip(inter[\"diffs\"], diffs):\n"
+     "        unanimous |= sign(dd_) == sd",
+     [P.pin_stats_example]),
+    ("stats_unanimous_skips_zero_differences", "        unanimous &= sign(dd_) == sd",
+     "        unanimous &= (sign(dd_) == sd) | (dd_ == 0)",
+     [P.pin_stats_example]),
+    ("stats_flips_vs_applied_sign", "flip_e = sign(u) != sd", "flip_e = sg != sd",
+     [P.pin_stats_example]),
+    ("stats_flips_vs_worker_sign", "flip_e = sign(u) != sd", "flip_e = sign(u) != sign(inter[\"diffs\"][0])",
+     [P.pin_worked_example, P.pin_stats_example]),
+    ("stats_zero_of_unrandomized_sign", "zero_e = sg == 0", "zero_e = sign(u) == 0",
+     [P.pin_stats_example]),
+    ("stats_delta_sq_of_u", "sq = delta[sel] ** 2", "sq = u[sel].astype(np.float64) ** 2",
+     [P.pin_worked_example]),
+    ("stats_clamp_inclusive", "clamp_e = (np.abs(u) > np.asarray(f32(B), dtype=u.dtype))",
+     "clamp_e = (np.abs(u) >= np.asarray(f32(B), dtype=u.dtype))",
+     [P.pin_stats_example]),
+    ("rsign_zero_inclusive", "return np.where(r < p, s, dt(0.0)).astype(u.dtype)",
+     "return np.where(r <= p, s, dt(0.0)).astype(u.dtype)",
+     [P.pin_stats_example]),
     ("stats_clamp_threshold", "clamp_e = (np.abs(u) > np.asarray(f32(B), dtype=u.dtype))",
      "clamp_e = (np.abs(u) > np.asarray(f32(B) / 2, dtype=u.dtype))",
      [P.pin_stats]),
