@@ -387,27 +387,31 @@ const char* dsm_last_error(void);
  * tiles of 1024 elements (a one-tensor model of up to 2^29 elements); larger
  * layouts return DSM_ERANGE.
  *
- * Arguments: layout, n (1..64) and hp as for dsm_create (only the global
- * fields of hp and its seed are used); gamma the round's gamma_t (> 0);
- * round the round index t (it keys the randomized sign); x and m the global
- * model and momentum (d fp32 each, device); replicas the n worker models
- * (device, fp32, worker i at replicas + i*replica_stride, replica_stride >= d
- * and a multiple of 8); x, m and replicas 16-byte aligned.  x, m and the
- * replicas are updated in place.  stats: NULL, or num_tensors entries in
- * device memory (stats_is_device = 1) or host memory (0; the call then
- * synchronises the stream).  Runs on the current device, which must own
- * the buffers.
+ * Arguments: layout, n (1..64) and hp as for dsm_create (the tensor list
+ * passes the same checks; of hp only the global fields and the seed are
+ * used, and global_mode must be DSM_GLOBAL_SIGN_MOMENTUM: the other global
+ * steps return DSM_EINVAL here); gamma the round's gamma_t (> 0); round the
+ * round index t (it keys the randomized sign); x and m the global model and
+ * momentum (d fp32 each); replicas the n worker models (fp32, worker i at
+ * replicas + i*replica_stride, replica_stride >= d and a multiple of 8);
+ * x, m and replicas 16-byte aligned, and device memory of the current
+ * device (checked: DSM_EINVAL otherwise).  x, m and the replicas are
+ * updated in place.  stats: NULL, or num_tensors entries in device memory
+ * of the current device (stats_is_device = 1) or in host memory (0; the
+ * call then copies them there and synchronises the stream).
  *
- * The first call on a device looks up the scratch array's device address
- * (cudaGetSymbolAddress) and caches it; make that first call before any
- * stream capture.  All calls share the one scratch array and leave their
- * contents in it; nothing in it needs to start at zero, because every call
- * rewrites the parts it reads.  Calls whose work overlaps on the GPU (on
- * different streams, or from different threads, on the same device) race
- * on the scratch array: order them on one stream or serialise them.  The
- * layout's tensor list is copied to the device on the stream; from pageable
- * host memory that copy has consumed the list when the call returns, from
- * pinned memory the list must stay unchanged until the stream reaches it. */
+ * Every call looks up the scratch array's device address on the current
+ * device (cudaGetSymbolAddress: a lookup, no allocation).  The first call
+ * on a device may load the library's device code there; make that first
+ * call before any stream capture.  All calls share the one scratch array
+ * and leave their contents in it; nothing in it needs to start at zero,
+ * because every call rewrites the parts it reads.  Calls whose work
+ * overlaps on the GPU (on different streams, or from different threads, on
+ * the same device) race on the scratch array: order them on one stream or
+ * serialise them.  The layout's tensor list is copied from host memory to
+ * the device on the stream; from pageable host memory that copy has
+ * consumed the list when the call returns, from pinned memory the list must
+ * stay unchanged until the stream reaches it. */
 #define DSM_NOALLOC_MAX_TENSORS 4096u
 #define DSM_NOALLOC_MAX_TILES   524288u
 #define DSM_NOALLOC_SCRATCH_BYTES 25657344u

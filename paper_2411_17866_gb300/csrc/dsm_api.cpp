@@ -73,7 +73,6 @@ struct ArenaLayout {
 
 int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp, ArenaLayout* al) {
     if (!layout || !hp) return fail(DSM_EINVAL, "layout and hparams must not be NULL");
-    if (layout->count == 0 || !layout->tensors) return fail(DSM_EINVAL, "layout has no tensors");
     if (n == 0) return fail(DSM_EINVAL, "n (workers) must be >= 1");
     if (n > kMaxWorkers) return fail(DSM_ERANGE, "n = %u exceeds the maximum of %u workers", n, kMaxWorkers);
     if (hp->base != DSM_BASE_ADAMW && hp->base != DSM_BASE_SGDM)
@@ -109,17 +108,8 @@ int check_layout_and_hp(const dsm_layout* layout, uint32_t n, const dsm_hparams*
         return fail(DSM_EINVAL, "unknown bits in hparams.flags");
 
     uint64_t d = 0, tiles = 0;
-    for (uint32_t i = 0; i < layout->count; ++i) {
-        const dsm_tensor& t = layout->tensors[i];
-        if (t.kind > DSM_KIND_LN_B) return fail(DSM_EINVAL, "tensor %u: kind %u unknown", i, t.kind);
-        if (!finite(t.grad_scale)) return fail(DSM_EINVAL, "tensor %u: grad_scale not finite", i);
-        if (t.reserved != 0) return fail(DSM_EINVAL, "tensor %u: reserved must be 0", i);
-        if (t.numel > kMaxD) return fail(DSM_ERANGE, "tensor %u: numel too large", i);
-        d += t.numel;
-        tiles += (t.numel + kTile - 1) / kTile;
-        if (d > kMaxD) return fail(DSM_ERANGE, "model larger than 2^40 elements");
-    }
-    if (d == 0) return fail(DSM_EINVAL, "the model has no elements (every tensor has numel 0)");
+    const int rc = check_tensor_list(layout, &d, &tiles);
+    if (rc != DSM_OK) return rc;
     if (tiles * n >= (1ull << 32)) return fail(DSM_ERANGE, "too many tiles (%llu) for n = %u", (unsigned long long)tiles, n);
 
     ArenaLayout a;
@@ -169,6 +159,25 @@ struct DeviceGuard {
 }  // namespace
 
 void dsm::set_last_error_message(const char* msg) { g_last_error = msg; }
+
+int dsm::check_tensor_list(const dsm_layout* layout, uint64_t* d_out, uint64_t* tiles_out) {
+    if (!layout || layout->count == 0 || !layout->tensors) return fail(DSM_EINVAL, "layout has no tensors");
+    uint64_t d = 0, tiles = 0;
+    for (uint32_t i = 0; i < layout->count; ++i) {
+        const dsm_tensor& t = layout->tensors[i];
+        if (t.kind > DSM_KIND_LN_B) return fail(DSM_EINVAL, "tensor %u: kind %u unknown", i, t.kind);
+        if (!finite(t.grad_scale)) return fail(DSM_EINVAL, "tensor %u: grad_scale not finite", i);
+        if (t.reserved != 0) return fail(DSM_EINVAL, "tensor %u: reserved must be 0", i);
+        if (t.numel > kMaxD) return fail(DSM_ERANGE, "tensor %u: numel too large", i);
+        d += t.numel;
+        tiles += (t.numel + kTile - 1) / kTile;
+        if (d > kMaxD) return fail(DSM_ERANGE, "model larger than 2^40 elements");
+    }
+    if (d == 0) return fail(DSM_EINVAL, "the model has no elements (every tensor has numel 0)");
+    *d_out = d;
+    *tiles_out = tiles;
+    return DSM_OK;
+}
 
 struct dsm_handle {
     int device = 0;

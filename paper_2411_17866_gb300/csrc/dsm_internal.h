@@ -7,6 +7,8 @@
 
 #include <cuda_runtime.h>
 
+#include "dsm.h"
+
 namespace dsm {
 
 // Elements of one tile.  A tile lies inside one tensor; a tensor of numel
@@ -150,5 +152,10 @@ cudaError_t launch_stats(const Problem& p, uint32_t producer_grid, cudaStream_t 
 
 // Sets the calling thread's message returned by dsm_last_error() (dsm_api.cpp).
 void set_last_error_message(const char* msg);
+
+// The checks every entry point applies to a tensor list (dsm_api.cpp): at least one tensor, kinds
+// known, grad_scale finite, reserved 0, sizes within 2^40 elements, and at least one element.
+// Sets *d and *tiles (tiles of kTile elements) and returns DSM_OK, or fails like every call.
+int check_tensor_list(const dsm_layout* layout, uint64_t* d, uint64_t* tiles);
 
 }  // namespace dsm

@@ -7,7 +7,7 @@
 // one static device array instead; this file allocates nothing.
 
 #include <cstdio>
-#include <mutex>
+#include <string>
 
 #include "dsm.h"
 #include "dsm_internal.h"
@@ -100,10 +100,6 @@ __global__ void __launch_bounds__(kThreads) k_noalloc_tile_table(unsigned char* 
     }
 }
 
-std::mutex g_mu;
-constexpr int kMaxDevices = 64;
-void* g_scratch_addr[kMaxDevices] = {};
-
 }  // namespace
 }  // namespace dsm
 
@@ -128,6 +124,24 @@ int na_cuda(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// DSM_OK if p is device (or managed) memory of device `dev`; the name goes into the message otherwise.
+int check_device_buffer(const void* p, int dev, const char* name) {
+    cudaPointerAttributes attr;
+    const cudaError_t err = cudaPointerGetAttributes(&attr, p);
+    if (err != cudaSuccess) {
+        cudaGetLastError();
+        char what[96];
+        snprintf(what, sizeof what, "cudaPointerGetAttributes(%s)", name);
+        return na_cuda(err, what);
+    }
+    if ((attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged) || attr.device != dev) {
+        char msg[128];
+        snprintf(msg, sizeof msg, "%s is not device memory of the current device", name);
+        return na_fail(DSM_EINVAL, msg);
+    }
+    return DSM_OK;
+}
+
 }  // namespace
 
 extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, const dsm_hparams* hp, float gamma,
@@ -135,7 +149,12 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
                                        uint64_t replica_stride, dsm_tensor_stats* stats, int stats_is_device,
                                        dsm_stream_t stream) {
     if (!layout || !hp || !x || !m || !replicas) return na_fail(DSM_EINVAL, "NULL argument");
-    if (layout->count == 0 || !layout->tensors) return na_fail(DSM_EINVAL, "layout has no tensors");
+    // the tensor list passes the same checks as in dsm_create()
+    uint64_t d = 0, tiles = 0;
+    if (const int rc = check_tensor_list(layout, &d, &tiles); rc != DSM_OK) {
+        const std::string why = dsm_last_error();
+        return na_fail(rc, why.c_str());
+    }
     if (layout->count > kNaMaxTensors) return na_fail(DSM_ERANGE, "more than DSM_NOALLOC_MAX_TENSORS (4096) tensors");
     if (n == 0 || n > kMaxWorkers) return na_fail(n == 0 ? DSM_EINVAL : DSM_ERANGE, "n must lie in [1, 64]");
     if (!(gamma > 0.f && gamma < 3.0e38f)) return na_fail(DSM_EINVAL, "gamma must be finite and > 0");
@@ -148,14 +167,6 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
         return na_fail(DSM_EINVAL, "only the sign-momentum global step (DSM_GLOBAL_SIGN_MOMENTUM) is available here");
     if (hp->sign_mode != DSM_SIGN && !(hp->rsign_B > 0.f && hp->rsign_B < 3.0e38f))
         return na_fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
-    uint64_t d = 0, tiles = 0;
-    for (uint32_t i = 0; i < layout->count; ++i) {
-        const uint64_t ne = layout->tensors[i].numel;
-        if (ne > (1ull << 40)) return na_fail(DSM_ERANGE, "tensor too large");
-        d += ne;
-        tiles += (ne + kTile - 1) / kTile;
-    }
-    if (d == 0) return na_fail(DSM_EINVAL, "the model has no elements");
     if (tiles > kNaMaxTiles)
         return na_fail(DSM_ERANGE, "layout needs more than DSM_NOALLOC_MAX_TILES (524288) tiles of 1024 elements");
     if (replica_stride < d || replica_stride % 8 != 0)
@@ -166,28 +177,18 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return na_cuda(err, "cudaGetDevice");
-    if (dev < 0 || dev >= kMaxDevices) return na_fail(DSM_ERANGE, "device index beyond 63");
-    cudaPointerAttributes attr;
-    err = cudaPointerGetAttributes(&attr, x);
-    if (err != cudaSuccess) {
-        cudaGetLastError();
-        return na_cuda(err, "cudaPointerGetAttributes(x)");
-    }
-    if ((attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged) || attr.device != dev)
-        return na_fail(DSM_EINVAL, "x is not device memory of the current device");
+    if (int rc = check_device_buffer(x, dev, "x"); rc != DSM_OK) return rc;
+    if (int rc = check_device_buffer(m, dev, "m"); rc != DSM_OK) return rc;
+    if (int rc = check_device_buffer(replicas, dev, "replicas"); rc != DSM_OK) return rc;
+    if (stats && stats_is_device)
+        if (int rc = check_device_buffer(stats, dev, "stats"); rc != DSM_OK) return rc;
 
-    // Set-up, once per device with that device current: the scratch array's device address.
+    // The scratch array's device address on the current device, looked up by every call (a lookup,
+    // no allocation), so that it is never stale: not after cudaDeviceReset, and not in another
+    // context.  The first call on a device may load the library's device code there.
     void* scratch_v = nullptr;
-    {
-        std::lock_guard<std::mutex> lock(g_mu);
-        if (!g_scratch_addr[dev]) {
-            void* p = nullptr;
-            err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-            if (err != cudaSuccess) return na_cuda(err, "cudaGetSymbolAddress(scratch)");
-            g_scratch_addr[dev] = p;
-        }
-        scratch_v = g_scratch_addr[dev];
-    }
+    err = cudaGetSymbolAddress(&scratch_v, g_noalloc_scratch);
+    if (err != cudaSuccess) return na_cuda(err, "cudaGetSymbolAddress(scratch)");
     unsigned char* scratch = static_cast<unsigned char*>(scratch_v);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
