@@ -12,8 +12,8 @@ Metric: params/s per global round = d x rounds / device time (whole job).
 Also reported: the dominant kernel's roofline (algorithmic bytes per launch
 over its CUDA-event duration, against the measured HBM copy bandwidth), an
 end-to-end figure through the C ABI with host gradient buffers, the SM
-clocks seen during the timed region, and the CPU oracle timed on a bounded
-sample of the same workload.
+clocks seen during the timed region, and the C++ CPU oracle timed on a
+bounded sample of the same workload.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload gpt2s] [--impl reference]
 
@@ -24,6 +24,7 @@ one JSON line.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -39,7 +40,9 @@ import workloads as W  # noqa: E402
 
 METRIC = "params/s per global round (τ local + sign-momentum step); % HBM roofline"
 UNIT = "params/s"
-CPU_SAMPLE_ELEMS = 1 << 22
+# the CPU oracle's samples: all host cores, and one thread (about 10-30 s of CPU work on the GPT-2 workloads)
+CPU_SAMPLE_ELEMS = 1 << 24
+CPU_ONE_CORE_ELEMS = 1 << 21
 # the sources of the local-step kernels (their arithmetic lives in the shared device header)
 KERNELS_SRC = [os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", f) for f in ("dsm_device.cuh", "dsm_local.cu")]
 
@@ -63,11 +66,16 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    # the five workloads' short CUDA-event runs (the line's "workloads" record)
+    ap.add_argument("--no-workloads", action="store_true")
     # smaller cases of a workload (profiling captures): fewer workers, fewer local steps, or a
     # prefix of the tensor list holding at most this many parameters
     ap.add_argument("--n-workers", type=int, default=None)
     ap.add_argument("--tau", type=int, default=None)
     ap.add_argument("--max-params", type=int, default=None)
+    # or one flat weight tensor of this many parameters (the workload's n, tau, hyper-parameters and the
+    # first tensor's gradient scale)
+    ap.add_argument("--flat-params", type=int, default=None)
     # the global step: Algorithm 1 (default) or a variant of the ablations
     ap.add_argument("--global-mode", default=None, choices=sorted(GLOBAL_MODES))
     # fused round (default): the last local step inside the global step, lazy replica reset
@@ -83,7 +91,6 @@ GLOBAL_MODES = {"sign_momentum": W.GLOBAL_SIGN_MOMENTUM, "slowmo": W.GLOBAL_SLOW
 
 
 def select_workload(args):
-    import dataclasses
     wl = W.WORKLOADS[args.workload]
     changes = {}
     notes = []
@@ -116,6 +123,9 @@ def select_workload(args):
             total += t.numel
         changes["tensors"] = tuple(keep)
         notes.append(f"reduced to the first {len(keep)} tensors ({total} params)")
+    if args.flat_params:
+        changes["tensors"] = W.flat_layout(args.flat_params, wl.tensors[0].grad_scale)
+        notes.append(f"one flat tensor of {args.flat_params} params")
     if changes:
         if notes:
             changes["name"] = wl.name + " [" + ", ".join(notes) + "]"
@@ -143,7 +153,6 @@ def max_over_ranks(seconds: float, world: int) -> float:
 
 def shard_hparams(hp, rank: int):
     """Each rank's parameter shard draws its own synthetic inputs (seed + rank)."""
-    import dataclasses
     return dataclasses.replace(hp, seed=hp.seed + rank)
 
 
@@ -291,73 +300,42 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(rows), "power_w_max": pmax, "gpu": self.gpu}
 
 
-def host_cores() -> int:
-    try:
-        return len(os.sched_getaffinity(0))
-    except AttributeError:
-        return os.cpu_count() or 1
-
-
-def _oracle_slice_worker(tensors, n, tau, hp, start, count, warmup, steps, barrier, out):
-    """One process of the all-cores oracle run: rounds over elements [start, start + count)."""
+def cxx_oracle_round(wl, count, threads, steps=1, warmup=0):
+    """The C++ oracle, as it stands, over elements [0, count) of the workload with `threads` OpenMP threads
+    (0: every host core): `warmup` untimed rounds, then the wall time of each of `steps` rounds."""
     import numpy as np
 
-    from oracle import dsm_oracle as O
-    ora = O.OracleRun(tensors, n, tau, hp, elems=np.arange(start, start + count, dtype=np.int64))
+    from oracle.cxx_oracle import CxxOracleRun
+    ora = CxxOracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64), threads=threads)
     for _ in range(warmup):
         ora.run_round()
-    for step in range(steps):
-        barrier.wait()
-        t0 = time.time()
-        ora.run_round()
-        out.put((step, t0, time.time()))
-
-
-def parallel_oracle(wl, per_worker, workers, steps=1, warmup=0):
-    """The CPU oracle, as it stands, in `workers` processes over consecutive element slices of
-    `per_worker` elements (every step is elementwise, so slices are independent).  Processes start
-    with spawn (the parent holds a CUDA context); a barrier starts each step in all of them, and a
-    step's time is the first start to the last finish.  Returns (elements, step wall times)."""
-    import multiprocessing as mp
-    ctx = mp.get_context("spawn")
-    per_worker = max(1, min(per_worker, wl.d // workers))
-    barrier, out = ctx.Barrier(workers), ctx.Queue()
-    procs = [ctx.Process(target=_oracle_slice_worker,
-                         args=(wl.tensors, wl.n, wl.tau, wl.hp, i * per_worker, per_worker, warmup, steps, barrier,
-                               out)) for i in range(workers)]
-    for p in procs:
-        p.start()
-    marks = [out.get() for _ in range(workers * steps)]
-    for p in procs:
-        p.join()
     walls = []
-    for step in range(steps):
-        t = [(a, b) for st, a, b in marks if st == step]
-        walls.append(max(b for _, b in t) - min(a for a, _ in t))
-    return per_worker * workers, walls
-
-
-def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, rounds=1):
-    """The CPU oracle, as it stands: one round over a contiguous sample of the workload on every host
-    core (one process per core, one slice each), and the same on one core."""
-    import numpy as np
-
-    from oracle import dsm_oracle as O
-    count = min(elems_count, wl.d)
-    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=np.arange(count, dtype=np.int64))
-    t0 = time.perf_counter()
-    for _ in range(rounds):
+    for _ in range(steps):
+        t0 = time.perf_counter()
         ora.run_round()
-    dt = time.perf_counter() - t0
-    one = {"value": count * rounds / dt, "cores": 1,
-           "sample": f"{rounds} round(s) over elements [0, {count}), one thread; {dt:.2f} s"}
-    cores = host_cores()
-    total, walls = parallel_oracle(wl, count, cores, steps=rounds)
-    return {"value": total * rounds / sum(walls), "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{rounds} round(s) (tau={wl.tau} local steps x n={wl.n} workers + global step) over "
-                      f"elements [0, {total}) of the {wl.d}-parameter layout, numpy fp32, {cores} processes "
-                      f"of {total // cores} consecutive elements each; {sum(walls):.2f} s",
-            "one_core": one}
+        walls.append(time.perf_counter() - t0)
+    return walls
+
+
+def oracle_threads() -> int:
+    from oracle.cxx_oracle import load
+    return int(load().dsmo_max_threads())
+
+
+def cpu_baseline(wl, elems_count=CPU_SAMPLE_ELEMS, one_core_count=CPU_ONE_CORE_ELEMS):
+    """The C++ oracle, as it stands: one round over a contiguous sample of the workload on every host core
+    (OpenMP over elements), and one round over a smaller sample on one thread."""
+    count = min(elems_count, wl.d)
+    one = min(one_core_count, wl.d)
+    cores = oracle_threads()
+    wall = cxx_oracle_round(wl, count, 0)[0]
+    wall1 = cxx_oracle_round(wl, one, 1)[0]
+    return {"value": count / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"1 round (tau={wl.tau} local steps x n={wl.n} workers + global step) over elements "
+                      f"[0, {count}) of the {wl.d}-parameter layout: the C++ oracle (g++ -O2 -ffp-contract=off), "
+                      f"OpenMP over elements on {cores} threads; {wall:.2f} s",
+            "one_core": {"value": one / wall1, "cores": 1,
+                         "sample": f"1 round over elements [0, {one}), one thread; {wall1:.2f} s"}}
 
 
 def run_reference(args):
@@ -366,20 +344,20 @@ def run_reference(args):
         return 0
     wl = select_workload(args)
     # each step one round over a contiguous sample, sized so that the whole run stays near a minute of
-    # CPU time whatever --steps and --warmup are (about 2^20 elements per step at the defaults)
-    per_step = (1 << 20) * (20 + 3) // max(1, args.steps + args.warmup)
+    # wall time whatever --steps and --warmup are (about 2^23 elements per step at the defaults)
+    per_step = (1 << 23) * (20 + 3) // max(1, args.steps + args.warmup)
     per_step = per_step * 48 // (wl.n * wl.tau)          # the defaults' n*tau is 48
-    count = int(min(max(per_step, 1 << 14), 1 << 22, wl.d))
-    cores = host_cores()
-    total, walls = parallel_oracle(wl, count, cores, steps=args.steps, warmup=args.warmup)
+    count = int(min(max(per_step, 1 << 14), 1 << 25, wl.d))
+    cores = oracle_threads()
+    walls = cxx_oracle_round(wl, count, 0, steps=args.steps, warmup=args.warmup)
     dt = sum(walls)
-    value = total * args.steps / dt
+    value = count * args.steps / dt
     sample = (f"each step: one round (tau={wl.tau} x n={wl.n} local steps + global step) over elements "
-              f"[0, {total}) of the {wl.d}-parameter layout; numpy fp32 oracle in {cores} processes of "
-              f"{total // cores} consecutive elements each")
+              f"[0, {count}) of the {wl.d}-parameter layout; the C++ oracle (g++ -O2 -ffp-contract=off), "
+              f"OpenMP over elements on {cores} threads")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": compute_dtype(wl),
             "data": "synthetic", "config": workload_config(wl, args.gpus),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -397,6 +375,143 @@ def workload_config(wl, gpus):
             "parallelism": f"param-shard x{gpus}" if gpus > 1 else "single GPU",
             "l2": "inputs larger than L2 (129 MB): each local-step launch streams "
                   f"{wl.n * wl.d * bytes_per_elem_local(wl) / 1e9:.1f} GB"}
+
+
+SPEC_HBM_GBS = 8000.0   # GB300's HBM3e figure (~8 TB/s) that the 80 % per-kernel target is stated against
+
+
+def round_events(run, wl, stream, t, tau, fused, lazy, reset, rec):
+    """Enqueue one global round; with `rec` (a dict of lists) bracket each launch with CUDA events on the
+    launching stream and record the algorithmic bytes of every local-step and global-step launch."""
+    import torch
+
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    for k in range(tau):
+        if rec is not None:
+            a, b = ev(), ev()
+            a.record(stream)
+            run.fill_synthetic_grads(t * tau + k, stream)
+            b.record(stream)
+            rec["fill"].append((a, b, 0))
+        else:
+            run.fill_synthetic_grads(t * tau + k, stream)
+        if rec is not None and not (fused and k == tau - 1):
+            a, b = ev(), ev()
+            a.record(stream)
+            run.local_step(stream)
+            b.record(stream)
+            # deferred reset: the first local step starts every worker from x (read once per tile);
+            # restarted base optimizer: the first local step reads no state
+            nbytes = local_step_bytes(wl, from_x=lazy and k == 0 and t > 0, zero_state=reset and k == 0 and t > 0)
+            rec["local"].append((a, b, nbytes))
+        else:
+            run.local_step(stream)
+    if rec is not None:
+        a, b = ev(), ev()
+        a.record(stream)
+        run.global_step(stream)
+        b.record(stream)
+        if fused:   # with tau = 1 the fused launch is also the round's first local step
+            first = tau == 1 and t > 0
+            gbytes = wl.d * bytes_per_param_fused_last(wl, from_x=first, zero_state=reset and first)
+        else:
+            gbytes = wl.d * bytes_per_param_global(wl, lazy)
+        rec["global"].append((a, b, gbytes))
+    else:
+        run.global_step(stream)
+
+
+def time_rounds(run, wl, stream, t, warmup, steps, world=1, sampler=None):
+    """W untimed rounds, then K rounds between CUDA events on the launching stream (barrier and
+    synchronize on both sides).  Returns the next round index and the per-kernel timings."""
+    import torch
+    import torch.distributed as dist
+    fused, lazy = fused_round_active(wl), lazy_reset_active(wl)
+    reset = bool(wl.hp.flags & W.FLAG_RESET_LOCAL_STATE)
+    for _ in range(warmup):
+        round_events(run, wl, stream, t, wl.tau, fused, lazy, reset, None)
+        t += 1
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+    rec = {"fill": [], "local": [], "global": []}
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        round_events(run, wl, stream, t, wl.tau, fused, lazy, reset, rec)
+        t += 1
+    end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    res = {"elapsed": max_over_ranks(start.elapsed_time(end) / 1e3, world), "clocks": clocks, "fused": fused,
+           "lazy": lazy}
+    for key, evs in rec.items():
+        res[key + "_ms"] = [a.elapsed_time(b) for a, b, _ in evs]
+        res[key + "_bytes"] = [nb for _, _, nb in evs]
+    return t, res
+
+
+def kernel_figures(wl, res, peak):
+    """Per-kernel achieved bandwidth (algorithmic bytes over CUDA-event time) against both peaks."""
+    local_ms, global_ms = res["local_ms"], res["global_ms"]
+    global_gbs = sum(res["global_bytes"]) / (sum(global_ms) / 1e3) / 1e9
+    out = {"global_gbs": global_gbs, "global_frac": global_gbs / peak, "global_spec_frac": global_gbs / SPEC_HBM_GBS,
+           "global_avg_ms": statistics.mean(global_ms), "global_bytes": statistics.mean(res["global_bytes"])}
+    if local_ms:
+        local_gbs = sum(res["local_bytes"]) / (sum(local_ms) / 1e3) / 1e9
+        out.update(local_gbs=local_gbs, local_frac=local_gbs / peak, local_spec_frac=local_gbs / SPEC_HBM_GBS,
+                   local_avg_ms=statistics.mean(local_ms), local_bytes=local_step_bytes(wl))
+    out["optimizer_only_value"] = wl.d * len(global_ms) / ((sum(local_ms) + sum(global_ms)) / 1e3)
+    return out
+
+
+def workload_sweep(dev, stream, peak, skip, steps=3, warmup=2):
+    """Every measured workload (fused round, as configured) timed briefly in this process with CUDA events:
+    params/s of the round and each kernel's fraction of both peaks.  `skip` maps a workload already timed
+    in this job to its figures."""
+    import torch
+
+    from paper_2411_17866_gb300 import dsm
+    out = {}
+    for key in ("flat1m", "gpt2s", "gpt2m", "gpt2l", "gpt2xl"):
+        if key in skip:
+            out[key] = skip[key]
+            continue
+        wl = W.WORKLOADS[key]
+        wl = dataclasses.replace(wl, hp=dataclasses.replace(wl.hp, flags=wl.hp.flags | W.FLAG_FUSED_ROUND))
+        run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, wl.hp, device=dev)
+        _, res = time_rounds(run, wl, stream, 0, warmup, steps)
+        run.close()
+        del run
+        torch.cuda.empty_cache()
+        out[key] = sweep_entry(wl, res, peak, steps)
+    return out
+
+
+def sweep_entry(wl, res, peak, steps):
+    f = kernel_figures(wl, res, peak)
+    e = {"params_per_s": wl.d * steps / res["elapsed"], "ms_per_round": res["elapsed"] / steps * 1e3,
+         "rounds_timed": steps, "optimizer_only_params_per_s": f["optimizer_only_value"],
+         "fused_last_plus_global_gbs": f["global_gbs"], "fused_last_plus_global_frac": f["global_frac"],
+         "fused_last_plus_global_frac_of_8tbs": f["global_spec_frac"],
+         "grad_fill_ms": statistics.mean(res["fill_ms"])}
+    if "local_gbs" in f:
+        e.update(local_step_gbs=f["local_gbs"], local_step_frac=f["local_frac"],
+                 local_step_frac_of_8tbs=f["local_spec_frac"])
+    return e
+
+
+def compute_dtype(wl) -> str:
+    """The arithmetic type of the path, with the gradients' storage type where it differs."""
+    return "f32 (bf16 grads)" if wl.hp.grad_dtype == W.BF16 else "f32"
 
 
 def main():
@@ -419,79 +534,9 @@ def main():
     stream = torch.cuda.current_stream(dev)
     tau = wl.tau
 
-    fused = fused_round_active(wl)
-    lazy = lazy_reset_active(wl)
-    reset = bool(wl.hp.flags & W.FLAG_RESET_LOCAL_STATE)
-    local_bytes = local_step_bytes(wl)
-
-    def round_(t, local_events=None, global_events=None, fill_events=None):
-        for k in range(tau):
-            if fill_events is not None:
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                run.fill_synthetic_grads(t * tau + k, stream)
-                b.record(stream)
-                fill_events.append((a, b))
-            else:
-                run.fill_synthetic_grads(t * tau + k, stream)
-            if local_events is not None and not (fused and k == tau - 1):
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                run.local_step(stream)
-                b.record(stream)
-                # deferred reset: the first local step starts every worker from x (read once per tile);
-                # restarted base optimizer: the first local step reads no state
-                nbytes = local_step_bytes(wl, from_x=lazy and k == 0 and t > 0, zero_state=reset and k == 0 and t > 0)
-                local_events.append((a, b, nbytes))
-            else:
-                run.local_step(stream)
-        if global_events is not None:
-            a = torch.cuda.Event(enable_timing=True)
-            b = torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            run.global_step(stream)
-            b.record(stream)
-            if fused:   # with tau = 1 the fused launch is also the round's first local step
-                first = tau == 1 and t > 0
-                gbytes = wl.d * bytes_per_param_fused_last(wl, from_x=first, zero_state=reset and first)
-            else:
-                gbytes = wl.d * bytes_per_param_global(wl, lazy)
-            global_events.append((a, b, gbytes))
-        else:
-            run.global_step(stream)
-
-    t = 0
-    for _ in range(args.warmup):
-        round_(t)
-        t += 1
-    torch.cuda.synchronize()
-
     sampler = ClockSampler(local) if (rank == 0 and not args.no_clocks) else None
-    if sampler:
-        sampler.start()
-    local_ev, global_ev, fill_ev = [], [], []
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for _ in range(args.steps):
-        round_(t, local_ev, global_ev, fill_ev)
-        t += 1
-    end.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    clocks = sampler.stop() if sampler else None
-    elapsed = max_over_ranks(start.elapsed_time(end) / 1e3, world)
-    local_ms = [a.elapsed_time(b) for a, b, _ in local_ev]
-    local_launch_bytes = [nb for _, _, nb in local_ev]
-    global_ms = [a.elapsed_time(b) for a, b, _ in global_ev]
-    global_launch_bytes = [nb for _, _, nb in global_ev]
-    fill_ms = [a.elapsed_time(b) for a, b in fill_ev]
+    t, res = time_rounds(run, wl, stream, 0, args.warmup, args.steps, world, sampler)
+    elapsed, clocks, fused, lazy = res["elapsed"], res["clocks"], res["fused"], res["lazy"]
 
     # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device
     # gradient copy + local step), the global step, and the new x read back to pinned host memory
@@ -528,6 +573,10 @@ def main():
                "steps": args.e2e_steps, "path": "dsm_local_step_host_grads (pinned host gradients, chunked "
                                                  "copies on a second stream) x tau, dsm_global_step, "
                                                  "dsm_read_params(x -> pinned host)"}
+        del host_g, host_x
+    run.close()
+    del run
+    torch.cuda.empty_cache()
 
     if rank != 0:
         if world > 1:
@@ -535,50 +584,59 @@ def main():
         return 0
 
     peak, peak_kind = measured_peaks()
-    # fused round: the last local step runs inside the global-step launch
-    global_bytes = statistics.mean(global_launch_bytes)
+    f = kernel_figures(wl, res, peak)
     grad_bytes = wl.n * wl.d * (2 if wl.hp.grad_dtype == W.BF16 else 4)
-    global_gbs = sum(global_launch_bytes) / (sum(global_ms) / 1e3) / 1e9
-    avg_global_s = statistics.mean(global_ms) / 1e3
-    if local_ms:   # the dominant kernel: the local step
-        avg_local_s = statistics.mean(local_ms) / 1e3
-        achieved = sum(local_launch_bytes) / (sum(local_ms) / 1e3) / 1e9
+    if "local_gbs" in f:   # the dominant kernel: the local step
+        achieved, avg_local_ms, local_bytes = f["local_gbs"], f["local_avg_ms"], f["local_bytes"]
         kname = "local_adamw" if wl.hp.base == W.BASE_ADAMW else "local_sgdm"
         # the traffic record holds for the workload as configured by default (a full local-step launch)
         default = wl.name == W.WORKLOADS[args.workload].name
         traffic = committed_traffic(f"{kname}:{args.workload}") if default else None
     else:          # tau = 1 in the fused round: the only launch is the fused last step + global step
-        avg_local_s, achieved, kname, traffic = avg_global_s, global_gbs, "fused_last_global", None
-        local_bytes = global_bytes
+        achieved, avg_local_ms, local_bytes = f["global_gbs"], f["global_avg_ms"], f["global_bytes"]
+        kname, traffic = "fused_last_global", None
     value = whole_job_value(wl.d, world, args.steps, elapsed)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": compute_dtype(wl), "data": "synthetic",
         "config": workload_config(wl, world),
         "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
+                     "spec_peak": SPEC_HBM_GBS, "spec_frac": achieved / SPEC_HBM_GBS,
                      "traffic": traffic, "algorithmic_bytes_per_launch": local_bytes,
-                     "avg_launch_ms": avg_local_s * 1e3},
-        "global_step": {"bytes_per_launch": global_bytes, "avg_ms": avg_global_s * 1e3,
-                        "achieved_gbs": global_gbs, "frac": global_gbs / peak,
+                     "avg_launch_ms": avg_local_ms},
+        "global_step": {"bytes_per_launch": f["global_bytes"], "avg_ms": f["global_avg_ms"],
+                        "achieved_gbs": f["global_gbs"], "frac": f["global_frac"], "spec_frac": f["global_spec_frac"],
                         "note": ("last local step fused with the global step, + statistics reduction"
                                  if fused else "fused global step + statistics reduction" +
                                  (" (replica reset deferred)" if lazy else "")) +
                                 ", CUDA events around both"},
-        "grad_fill": {"avg_ms": statistics.mean(fill_ms), "bytes_written_per_launch": grad_bytes,
-                      "write_gbs": grad_bytes / (statistics.mean(fill_ms) / 1e3) / 1e9,
+        "grad_fill": {"avg_ms": statistics.mean(res["fill_ms"]), "bytes_written_per_launch": grad_bytes,
+                      "write_gbs": grad_bytes / (statistics.mean(res["fill_ms"]) / 1e3) / 1e9,
                       "note": "synthetic gradients (stand-in for the backward pass); bound by instruction "
                               "issue of the SplitMix64 hash"},
-        "optimizer_only_value": wl.d * args.steps / ((sum(local_ms) + sum(global_ms)) / 1e3),
+        "optimizer_only_value": f["optimizer_only_value"],
         "gpu_launches": args.steps * (2 * tau + (1 if fused else 2)),
         "e2e": e2e,
         "clocks": clocks,
     }
+    if not args.no_workloads and world == 1:
+        sampler = ClockSampler(local) if not args.no_clocks else None
+        if sampler:
+            sampler.start()
+        done = {}
+        if wl.name == W.WORKLOADS[args.workload].name and fused:
+            done[args.workload] = sweep_entry(wl, res, peak, args.steps)
+        sweep = workload_sweep(dev, stream, peak, done)
+        line["workloads"] = {"note": "each workload's fused round as configured, timed in this job with CUDA "
+                                     "events (2 untimed + 3 timed rounds; the bench workload's entry is the "
+                                     "timed region above); fractions of the measured copy peak and of 8 TB/s; "
+                                     "flat1m's launches (50-117 MB) fit in L2",
+                             "clocks": sampler.stop() if sampler else None, **sweep}
     if not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(wl)
     print(json.dumps(line), flush=True)
-    run.close()
     if world > 1:
         dist.destroy_process_group()
     return 0

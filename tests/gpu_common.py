@@ -78,4 +78,7 @@ def sample_elements(tensors, count, seed=0, edge=64):
         if b > a:
             parts.append(np.arange(a, min(b, a + edge)))
             parts.append(np.arange(max(a, b - edge), b))
-    return np.unique(np.concatenate(parts)).astype(np.int64)
+    v = np.sort(np.concatenate(parts).astype(np.int64))   # sorted, then duplicates dropped
+    keep = np.ones(v.size, dtype=bool)
+    keep[1:] = v[1:] != v[:-1]
+    return v[keep]

@@ -99,9 +99,12 @@ def test_workload_selection_names_only_changes():
     import argparse
     import bench
     args = argparse.Namespace(workload="gpt2s", n_workers=None, tau=None, global_mode=None, fused=True,
-                              reset_local_state=False, max_params=None)
+                              reset_local_state=False, max_params=None, flat_params=None)
     import workloads as W
     assert bench.select_workload(args).name == W.WORKLOADS["gpt2s"].name
     args.tau, args.reset_local_state = 2, True
     name = bench.select_workload(args).name
     assert "tau=2" in name and "restarted" in name
+    args.flat_params = 1000
+    wl = bench.select_workload(args)
+    assert wl.d == 1000 and len(wl.tensors) == 1 and "flat tensor of 1000" in wl.name

@@ -19,6 +19,7 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 from oracle import dsm_oracle as O  # noqa: E402
+from oracle.cxx_oracle import CxxOracleRun  # noqa: E402
 from paper_2411_17866_gb300 import dsm  # noqa: E402
 
 
@@ -259,6 +260,40 @@ def test_deterministic_statistics():
     assert outs[0] == outs[1]
 
 
+def test_statistics_of_the_hand_built_global_step():
+    """The hand-computed d = 8, n = 3 global step (tests/golden/stats_example_d8.json, deterministic sign)
+    through the C ABI: one plain-SGD local step on zero gradients leaves every replica at x = 0, the
+    replicas and m are then set to the example's values, and the global step must give the hand-computed
+    x', m' and statistics exactly (every value is dyadic)."""
+    import json
+    import os
+    from fractions import Fraction
+    ex = json.load(open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "stats_example_d8.json")))
+    hpj = ex["hparams"]
+    fr = lambda v: float(Fraction(v))  # noqa: E731
+    hp = W.HParams(base=W.BASE_SGDM, lr=fr(hpj["gamma"]), mu=0.0, wd=0.0, g_b1=fr(hpj["beta1"]),
+                   g_b2=fr(hpj["beta2"]), g_eta=fr(hpj["eta"]), g_wd=fr(hpj["lambda"]), sign_mode=W.SIGN)
+    tensors = (W.Tensor("t", 8, W.KIND_WEIGHT, 1.0),)
+    vec = lambda vals: torch.tensor([fr(v) for v in vals], dtype=torch.float32)  # noqa: E731
+    run = dsm.DistributedSignMomentum(tensors, hpj["n"], 1, hp, x0=vec(ex["x"]))
+    run.load_grads(torch.zeros(hpj["n"], 8, dtype=torch.float32))
+    run.local_step()
+    for i, di in enumerate(ex["diffs"]["values"]):
+        run.write(dsm.BUF_REPLICA, vec(ex["x"]) - vec(di), worker=i)
+    run.write(dsm.BUF_M, vec(ex["m"]))
+    st = run.global_step(with_stats=True)[0]
+    torch.cuda.synchronize()
+    want = ex["modes"]["sign"]
+    sg = vec(want["sign"])
+    assert torch.equal(run.read(dsm.BUF_X), -fr(hpj["eta"]) * fr(hpj["gamma"]) * sg)
+    assert torch.equal(run.read(dsm.BUF_M), vec(ex["m_new"]))
+    for key in ("delta_sq", "drift"):
+        assert st[key] == fr(want["stats"][key]), key
+    for key in ("zero_sign", "flips", "unanimous", "clamped"):
+        assert st[key] == want["stats"][key], key
+    run.close()
+
+
 def test_x0_from_device_and_host():
     tensors, n, tau = MINI, 2, 1
     d = sum(t.numel for t in tensors)
@@ -273,22 +308,42 @@ def test_x0_from_device_and_host():
         run.close()
 
 
-@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
-@pytest.mark.parametrize("key", list(W.WORKLOADS))
+# The element-subset pin at full size: 10^7 random elements plus the first and last 4096 of every tensor.
+FULL_SAMPLE, FULL_EDGE = 10_000_000, 4096
+_FULL_ORACLE = {}
+
+
+def _full_oracle(key):
+    """The C++ oracle over the sampled elements of a full-size workload, through all of its rounds: x and m
+    after every round and the final state (computed once per workload: the fused and the unfused round
+    give the same results)."""
+    if key not in _FULL_ORACLE:
+        wl = W.WORKLOADS[key]
+        elems = None if wl.d <= (1 << 20) else sample_elements(wl.tensors, FULL_SAMPLE, edge=FULL_EDGE)
+        ora = CxxOracleRun(wl.tensors, wl.n, wl.tau, wl.hp, elems=elems, with_stats=elems is None)
+        per_round = []
+        for _ in range(wl.rounds):
+            ora.run_round()
+            per_round.append((ora.x.copy(), ora.m.copy(), ora.last_stats))
+        _FULL_ORACLE[key] = (elems, ora, per_round)
+    return _FULL_ORACLE[key]
+
+
+FULL_CASES = [(key, fused) for key in W.WORKLOADS for fused in (False, True)]
+
+
+@pytest.mark.parametrize("key,fused", FULL_CASES, ids=[f"{k}-{'fused' if f else 'unfused'}" for k, f in FULL_CASES])
 def test_full_workloads_sampled(key, fused):
-    """Each measured workload at full size, one round, in the launch sequence the benchmark uses,
-    checked on sampled elements against the element-subset oracle (first and last 64 elements of
-    every tensor plus 20000 random ones; the whole model for the flat workload)."""
+    """Each measured workload at full size through all of its rounds (5 for GPT-2 S and M, 3 for L, XL
+    and the flat workload), in the launch sequence the benchmark uses, fused and unfused, against the C++
+    oracle on sampled elements (10^7 random ones plus the first and last 4096 of every tensor; the whole
+    model for the flat workload): x and m after every round, every replica and optimizer state after the
+    last, bit for bit.  This reaches the round-keyed Philox draws at t > 0, AdamW's bias corrections at
+    j > tau and the first local step from x after a deferred reset at full size."""
     wl = W.WORKLOADS[key]
     hp = dataclasses.replace(wl.hp, flags=W.FLAG_FUSED_ROUND if fused else 0)
+    elems, ora, per_round = _full_oracle(key)
     run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp)
-    elems = None if wl.d <= (1 << 20) else sample_elements(wl.tensors, 20000)
-    ora = O.OracleRun(wl.tensors, wl.n, wl.tau, hp, elems=elems, with_stats=elems is None)
-    rounds = wl.rounds if elems is None else 1
-    for _ in range(rounds):
-        stats = run.synthetic_round(with_stats=True)
-        ora.run_round()
-    torch.cuda.synchronize()
     sel = None if elems is None else torch.from_numpy(elems).cuda()
     buf = torch.empty(wl.d, dtype=torch.float32, device="cuda")
 
@@ -296,22 +351,25 @@ def test_full_workloads_sampled(key, fused):
         run.read(which, i, out=buf)
         return (buf if sel is None else buf[sel]).cpu().numpy()
 
-    assert_bitexact(rd(dsm.BUF_X), ora.x, "x")
-    assert_bitexact(rd(dsm.BUF_M), ora.m, "m")
+    for t, (x_t, m_t, stats_t) in enumerate(per_round):
+        stats = run.synthetic_round(with_stats=True)
+        assert_bitexact(rd(dsm.BUF_X), x_t, f"x after round {t}")
+        assert_bitexact(rd(dsm.BUF_M), m_t, f"m after round {t}")
+        if elems is None:
+            compare_stats(stats, stats_t, wl.n)
+        else:   # properties that hold at any size
+            assert sum(s["unanimous"] for s in stats) <= wl.d
+            assert all(s["delta_sq"] > 0 for s in stats)
     for i in range(wl.n):
         assert_bitexact(rd(dsm.BUF_REPLICA, i), ora.X[i], f"replica {i}")
         assert_bitexact(rd(dsm.BUF_OPT_M, i), ora.opt_m[i], f"opt_m {i}")
         if ora.opt_v is not None:
             assert_bitexact(rd(dsm.BUF_OPT_V, i), ora.opt_v[i], f"opt_v {i}")
-    if elems is None:
-        compare_stats(stats, ora.last_stats, wl.n)
-    else:
-        # properties that hold at any size
-        assert sum(s["unanimous"] for s in stats) <= wl.d
-        assert all(s["delta_sq"] > 0 for s in stats)
     run.close()
-    del run
+    del run, buf
     torch.cuda.empty_cache()
+    if fused:
+        _FULL_ORACLE.pop(key, None)
 
 
 @pytest.mark.parametrize("key", list(W.WORKLOADS))
