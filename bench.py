@@ -17,9 +17,10 @@ bounded sample of the same workload.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload gpt2s] [--impl reference]
 
-Under torchrun each rank runs its own parameter shard of the workload's size
-(the path is elementwise, so a shard needs no communication); rank 0 prints
-one JSON line.
+Under torchrun rank r of G runs shard r of one model made of G copies of
+the workload's tensor list (d parameters per rank, starting at element r*d);
+the path is elementwise, so the shards need no communication, and rank 0
+prints one JSON line.
 """
 from __future__ import annotations
 
@@ -151,9 +152,13 @@ def max_over_ranks(seconds: float, world: int) -> float:
     return float(t.item())
 
 
-def shard_hparams(hp, rank: int):
-    """Each rank's parameter shard draws its own synthetic inputs (seed + rank)."""
-    return dataclasses.replace(hp, seed=hp.seed + rank)
+def rank_shard(wl, world: int, rank: int):
+    """Rank r's part of the weak-scaling model: `world` copies of the workload's tensor list, cut into
+    `world` contiguous shards of d parameters (shard r is copy r and starts at element r*d of that model).
+    Every step is elementwise, so the shards need no communication; together they compute exactly the
+    one-process run of the whole model."""
+    from paper_2411_17866_gb300.shard import repeated_model, shard_layout
+    return shard_layout(repeated_model(wl.tensors, world), world, rank)
 
 
 def whole_job_value(d_per_rank: int, world: int, rounds: int, seconds: float) -> float:
@@ -372,7 +377,8 @@ def workload_config(wl, gpus):
             "sign": ["sign", "rand-sign-2", "rand-sign-1"][wl.hp.sign_mode],
             "global_step": {v: k for k, v in GLOBAL_MODES.items()}[wl.hp.global_mode],
             "fused_round": bool(wl.hp.flags & W.FLAG_FUSED_ROUND),
-            "parallelism": f"param-shard x{gpus}" if gpus > 1 else "single GPU",
+            "parallelism": (f"parameter shards x{gpus}: rank r holds elements [r*d, (r+1)*d) of {gpus} copies "
+                            "of the tensor list, no collective on the data path") if gpus > 1 else "single GPU",
             "l2": "inputs larger than L2 (129 MB): each local-step launch streams "
                   f"{wl.n * wl.d * bytes_per_elem_local(wl) / 1e9:.1f} GB"}
 
@@ -529,8 +535,9 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     wl = select_workload(args)
-    hp = shard_hparams(wl.hp, rank)
-    run = dsm.DistributedSignMomentum(wl.tensors, wl.n, wl.tau, hp, device=dev)
+    shard = rank_shard(wl, world, rank)
+    run = dsm.DistributedSignMomentum(shard.tensors, wl.n, wl.tau, wl.hp, device=dev,
+                                      first_element=shard.first_element)
     stream = torch.cuda.current_stream(dev)
     tau = wl.tau
 
@@ -617,6 +624,8 @@ def main():
                       "note": "synthetic gradients (stand-in for the backward pass); bound by instruction "
                               "issue of the SplitMix64 hash"},
         "optimizer_only_value": f["optimizer_only_value"],
+        # per round: tau gradient fills, tau local steps (tau - 1 in the fused round), the global step and
+        # the statistics reduction
         "gpu_launches": args.steps * (2 * tau + (1 if fused else 2)),
         "e2e": e2e,
         "clocks": clocks,

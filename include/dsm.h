@@ -146,9 +146,19 @@ typedef struct {
     uint32_t reserved;    /* must be 0 */
 } dsm_tensor;
 
+/* A parameter layout: the tensor list, packed in order.  first_element is
+ * the logical index of the layout's first element within a larger model of
+ * which this layout is a contiguous part (0 for a whole model): a parameter
+ * shard of a model split over processes or GPUs (every step of Algorithm 1
+ * is elementwise, so a shard needs no communication).  The synthetic
+ * generators and the randomized sign's Philox counter then take element e
+ * of this layout as element first_element + e of the larger model, so the
+ * shards together compute exactly what one process computes on the whole
+ * model.  Must be a multiple of 4 and below 2^60 (DSM_EINVAL otherwise). */
 typedef struct {
     const dsm_tensor* tensors;  /* host array of count entries */
     uint32_t count;
+    uint64_t first_element;
 } dsm_layout;
 
 /* Hyper-parameters.  Float fields are used as the fp32 values given. */

@@ -80,7 +80,7 @@ def load() -> ctypes.CDLL:
     fp = POINTER(c_float)
     lib.dsmo_create.restype = c_void_p
     lib.dsmo_create.argtypes = [POINTER(dsmo_tensor), c_uint32, c_uint32, POINTER(dsmo_hparams), POINTER(c_int64),
-                                c_uint64, c_int]
+                                c_uint64, c_uint64, c_int]
     lib.dsmo_destroy.argtypes = [c_void_p]
     lib.dsmo_init_x0.argtypes = [c_void_p, fp]
     lib.dsmo_synthetic_grad.argtypes = [c_void_p, c_uint64, c_uint32, fp]
@@ -140,11 +140,11 @@ def bf16_round(v: float) -> float:
 class CxxOracleRun:
     """Algorithm 1 over a set of elements of one parameter layout, computed by the C++ oracle.
 
-    Same arguments and attributes as the numpy oracle's OracleRun (float32 only), plus ``threads``
-    (0: OpenMP's default).  X, opt_m and opt_v are [n][count] arrays (row i is worker i).
+    Same arguments and attributes as the numpy oracle's OracleRun (float32 only, first_element
+    included), plus ``threads`` (0: OpenMP's default).  X, opt_m and opt_v are [n][count] arrays (row i is worker i).
     """
 
-    def __init__(self, tensors, n, tau, hp, elems=None, x0=None, with_stats=False, threads=0):
+    def __init__(self, tensors, n, tau, hp, elems=None, x0=None, with_stats=False, threads=0, first_element=0):
         lib = load()
         self.tensors = list(tensors)
         self.n, self.tau, self.hp = int(n), int(tau), hp
@@ -158,7 +158,8 @@ class CxxOracleRun:
             arr[i].kind, arr[i].wd = int(t.kind), int(getattr(t, "wd", 1))
         self._hp = make_hparams(hp)
         self._ctx = lib.dsmo_create(arr, len(self.tensors), self.n, ctypes.byref(self._hp),
-                                    self.elems.ctypes.data_as(POINTER(c_int64)), self.count, int(threads))
+                                    self.elems.ctypes.data_as(POINTER(c_int64)), self.count, int(first_element),
+                                    int(threads))
         if not self._ctx:
             raise ValueError("an element index lies outside the model")
         self.x = np.empty(self.count, dtype=np.float32)

@@ -184,7 +184,7 @@ struct dsmo_problem {
     uint32_t n, num_tensors;
     dsmo_hparams hp;
     uint64_t count;
-    std::vector<uint64_t> elem;
+    std::vector<uint64_t> elem;  // index in the larger model (first_element + logical index)
     std::vector<uint32_t> tensor;
     std::vector<float> scale, scale2;
     std::vector<uint32_t> kind, wd;
@@ -192,9 +192,12 @@ struct dsmo_problem {
 };
 
 // The problem over elements elems[0..count) (logical indices into the packed tensor list; each must lie
-// inside the model).  threads <= 0: OpenMP's default.  Returns NULL if an element lies outside the model.
+// inside the model).  first_element: the layout's first element within a larger model of which it is a
+// contiguous part (a parameter shard); the generators and the Philox counter take element e as element
+// first_element + e of that model (0 for a whole model).  threads <= 0: OpenMP's default.  Returns NULL
+// if an element lies outside the model.
 dsmo_problem* dsmo_create(const dsmo_tensor* tensors, uint32_t num_tensors, uint32_t n, const dsmo_hparams* hp,
-                          const int64_t* elems, uint64_t count, int threads) {
+                          const int64_t* elems, uint64_t count, uint64_t first_element, int threads) {
     std::vector<uint64_t> starts(num_tensors + 1, 0);
     for (uint32_t T = 0; T < num_tensors; ++T) starts[T + 1] = starts[T] + tensors[T].numel;
     dsmo_problem* p = new dsmo_problem();
@@ -218,7 +221,7 @@ dsmo_problem* dsmo_create(const dsmo_tensor* tensors, uint32_t num_tensors, uint
         // the tensor holding e: the last one whose start is <= e (empty tensors hold nothing)
         const uint32_t T = static_cast<uint32_t>(
             std::upper_bound(starts.begin(), starts.end(), static_cast<uint64_t>(e)) - starts.begin() - 1);
-        p->elem[k] = static_cast<uint64_t>(e);
+        p->elem[k] = first_element + static_cast<uint64_t>(e);  // its index in the larger model
         p->tensor[k] = T;
         p->scale[k] = tensors[T].grad_scale;
         p->scale2[k] = 0.1f * tensors[T].grad_scale;

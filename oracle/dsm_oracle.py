@@ -462,6 +462,10 @@ class OracleRun:
     elems: logical element indices to simulate (None = all of them).
     x0: initial model on those elements (None = the hash initialisation).
     dtype: np.float32 (canonical) or np.float64 (twin).
+    first_element: the layout's first element within a larger model of
+    which it is a contiguous part (a parameter shard); the synthetic draws
+    and the randomized sign take element e as element first_element + e of
+    that model.  0 for a whole model.
 
     Worker optimizer states persist across rounds and are never averaged;
     only the model is synchronised (Algorithm 1, last step).  AdamW's step
@@ -472,7 +476,7 @@ class OracleRun:
     """
 
     def __init__(self, tensors, n, tau, hp, elems=None, x0=None, dtype=np.float32,
-                 with_stats=False):
+                 with_stats=False, first_element=0):
         self.tensors = list(tensors)
         self.n, self.tau, self.hp = int(n), int(tau), hp
         self.dt = np.dtype(dtype)
@@ -483,6 +487,9 @@ class OracleRun:
             elems = np.arange(self.d, dtype=np.int64)
         self.elems = np.asarray(elems, dtype=np.int64)
         self.tensor_of = np.searchsorted(self.starts, self.elems, side="right") - 1
+        # the elements' indices in the larger model that the layout is a part of: the generators and the
+        # randomized sign's counter use them (first_element = 0 for a whole model)
+        self.gidx = self.elems + np.int64(first_element)
         self.scale = np.array([t.grad_scale for t in self.tensors], dtype=np.float32)[self.tensor_of]
         kinds = np.array([t.kind for t in self.tensors])[self.tensor_of]
         wdflag = np.array([t.wd for t in self.tensors])[self.tensor_of] != 0
@@ -490,7 +497,7 @@ class OracleRun:
         self.wd_local = np.where(wdflag, T(f32(hp.wd)), T(0.0)).astype(self.dt)
         self.wd_global = np.where(wdflag, T(f32(hp.g_wd)), T(0.0)).astype(self.dt)
         if x0 is None:
-            x0 = init_x0(self.elems, kinds, hp.seed)
+            x0 = init_x0(self.gidx, kinds, hp.seed)
         self.x = np.asarray(x0).astype(self.dt)
         self.m = np.zeros_like(self.x)
         self.X = [self.x.copy() for _ in range(self.n)]
@@ -507,7 +514,7 @@ class OracleRun:
         self.last_inter = None
 
     def grads(self, step: int, worker: int) -> np.ndarray:
-        return synthetic_grad(self.elems, self.scale, self.hp.seed, step, worker, self.hp.grad_dtype)
+        return synthetic_grad(self.gidx, self.scale, self.hp.seed, step, worker, self.hp.grad_dtype)
 
     def local_step(self, grads=None):
         """Local step k of the current round for every worker, Eq. (local-steps)."""
@@ -533,7 +540,7 @@ class OracleRun:
         if mode == GLOBAL_SIGN_MOMENTUM:
             r = None
             if hp.sign_mode != 0:
-                r = philox_uniform(self.elems, hp.seed, self.t)
+                r = philox_uniform(self.gidx, hp.seed, self.t)
             x_new, m_new, inter = global_step(self.x, self.m, self.X, self.gamma, hp.g_b1, hp.g_b2,
                                               hp.g_eta, self.wd_global, hp.sign_mode, hp.rsign_B, r, self.dt)
         elif mode == GLOBAL_SLOWMO:

@@ -59,6 +59,14 @@ uint64_t draw_key(uint64_t seed, uint64_t stream, uint64_t idx) {
     return sm64_finalise(seed + j * 0x9E3779B97F4A7C15ull);
 }
 
+// The key of the same family for a layout that starts at element first_element (even) of a larger
+// model: element e of the layout takes output (first_element + e)/2 + 1 = e/2 + 1 + first_element/2
+// of the family, and output j of a generator seeded with `key` is the finaliser of key + j * gamma,
+// so moving the key by (first_element/2) * gamma moves every output index by first_element/2.
+uint64_t shard_key(uint64_t key, uint64_t first_element) {
+    return key + (first_element >> 1) * 0x9E3779B97F4A7C15ull;
+}
+
 bool finite(float v) { return std::isfinite(v); }
 
 // The arena: every region starts on a 256-byte boundary.
@@ -174,6 +182,8 @@ int dsm::check_tensor_list(const dsm_layout* layout, uint64_t* d_out, uint64_t* 
         if (d > kMaxD) return fail(DSM_ERANGE, "model larger than 2^40 elements");
     }
     if (d == 0) return fail(DSM_EINVAL, "the model has no elements (every tensor has numel 0)");
+    if (layout->first_element % 4 != 0 || layout->first_element >= (1ull << 60))
+        return fail(DSM_EINVAL, "first_element must be a multiple of 4 below 2^60");
     *d_out = d;
     *tiles_out = tiles;
     return DSM_OK;
@@ -207,6 +217,7 @@ struct dsm_handle {
     AdamScalars pending_a{};
     SgdmScalars pending_sa{};
     uint64_t j = 0;        // AdamW step count of the last local step (restarts each round with the reset flag)
+    uint64_t first_element = 0;  // the layout's first element within a larger model (a parameter shard)
     // local steps with host gradients (dsm_local_step_host_grads): chunk c covers tiles
     // [chunk_tile[c], chunk_tile[c+1]); ev_copied[c] marks its gradients in the arena
     std::vector<uint32_t> chunk_tile;
@@ -430,6 +441,7 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
     h->arena = static_cast<char*>(dev_arena);
     h->gamma = hp->lr;
     h->reset_local = (hp->flags & DSM_FLAG_RESET_LOCAL_STATE) != 0;
+    h->first_element = layout->first_element;
 
     // tensor and tile tables
     h->tensors.resize(al.num_tensors);
@@ -509,7 +521,8 @@ int dsm_create(const dsm_layout* layout, uint32_t n, uint32_t tau, const dsm_hpa
                                    s)) != cudaSuccess)
             return bail(err, "copy x0");
     }
-    if ((err = launch_init(p, h->shape, draw_key(hp->seed, 2, 0), x0 ? 0 : 1, s)) != cudaSuccess)
+    if ((err = launch_init(p, h->shape, shard_key(draw_key(hp->seed, 2, 0), h->first_element), x0 ? 0 : 1, s)) !=
+        cudaSuccess)
         return bail(err, "launch init");
     *out = h;
     return DSM_OK;
@@ -526,8 +539,9 @@ int dsm_set_gamma(dsm_handle* h, float gamma) {
 int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream) {
     if (!h) return fail(DSM_EINVAL, "handle is NULL");
     GradKeys k;
-    k.step = draw_key(h->hp.seed, 0, step);
-    for (uint32_t i = 0; i < kMaxWorkers; ++i) k.worker[i] = i < h->n ? draw_key(h->hp.seed, 1, i) : 0;
+    k.step = shard_key(draw_key(h->hp.seed, 0, step), h->first_element);
+    for (uint32_t i = 0; i < kMaxWorkers; ++i)
+        k.worker[i] = i < h->n ? shard_key(draw_key(h->hp.seed, 1, i), h->first_element) : 0;
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     int rc = materialize_pending(h, S(stream));
@@ -669,6 +683,7 @@ int dsm_global_step(dsm_handle* h, dsm_stream_t stream, dsm_tensor_stats* stats,
     g.mode = h->hp.global_mode;
     g.philox_k0 = static_cast<uint32_t>(h->hp.seed & 0xFFFFFFFFull);
     g.philox_k1 = static_cast<uint32_t>(h->t & 0xFFFFFFFFull);
+    g.philox_q0 = h->first_element >> 2;
     cudaStream_t s = S(stream);
     cudaError_t err;
     uint32_t grid = 0;  // CTAs of the global-step launch (the statistics reduction needs it)

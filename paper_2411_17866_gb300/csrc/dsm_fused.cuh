@@ -166,7 +166,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
             }
             float ru[4] = {0.f, 0.f, 0.f, 0.f};
             if (kGlobal == kGlobalSign && g.sign_mode != 0) {
-                const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                const uint4 b = philox_block((gi >> 2) + g.philox_q0, g.philox_k0, g.philox_k1);
                 ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
             }
 #pragma unroll
@@ -210,7 +210,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
                 }
                 float r = 0.f;
                 if (kGlobal == kGlobalSign && g.sign_mode != 0)
-                    r = philox_unit(word_of(philox_block(gj >> 2, g.philox_k0, g.philox_k1), gj & 3));
+                    r = philox_unit(word_of(philox_block((gj >> 2) + g.philox_q0, g.philox_k0, g.philox_k1), gj & 3));
                 if (kGlobal == kGlobalRuntime) {
                     global_elem_rt<NW>(x, m, d, g, lam_g, r, st);
                 } else if (kGlobal == kGlobalAdamW) {

@@ -106,6 +106,7 @@ struct GlobalScalars {
     int sign_mode;
     int mode;              // DSM_GLOBAL_*: read by the fused round's kernel for the ablation variants
     uint32_t philox_k0, philox_k1;
+    uint64_t philox_q0;    // counter of the layout's first element group: first_element / 4
     int skip_reset;        // K4: leave the replicas' reset to x pending (the next local step starts from x)
 };
 
@@ -154,7 +155,8 @@ cudaError_t launch_stats(const Problem& p, uint32_t producer_grid, cudaStream_t 
 void set_last_error_message(const char* msg);
 
 // The checks every entry point applies to a tensor list (dsm_api.cpp): at least one tensor, kinds
-// known, grad_scale finite, reserved 0, sizes within 2^40 elements, and at least one element.
+// known, grad_scale finite, reserved 0, sizes within 2^40 elements, at least one element, and
+// first_element a multiple of 4 below 2^60.
 // Sets *d and *tiles (tiles of kTile elements) and returns DSM_OK, or fails like every call.
 int check_tensor_list(const dsm_layout* layout, uint64_t* d, uint64_t* tiles);
 

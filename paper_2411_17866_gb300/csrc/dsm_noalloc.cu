@@ -230,6 +230,7 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     g.sign_mode = hp->sign_mode;
     g.philox_k0 = static_cast<uint32_t>(hp->seed & 0xFFFFFFFFull);
     g.philox_k1 = static_cast<uint32_t>(round & 0xFFFFFFFFull);
+    g.philox_q0 = layout->first_element >> 2;
     uint32_t grid = 0;
     if ((err = launch_global(p, ls, g, s, &grid)) != cudaSuccess) return na_cuda(err, "launch global step");
     if ((err = launch_stats(p, grid, s)) != cudaSuccess) return na_cuda(err, "launch statistics");

@@ -46,7 +46,7 @@ class dsm_tensor(ctypes.Structure):
 
 
 class dsm_layout(ctypes.Structure):
-    _fields_ = [("tensors", POINTER(dsm_tensor)), ("count", c_uint32)]
+    _fields_ = [("tensors", POINTER(dsm_tensor)), ("count", c_uint32), ("first_element", c_uint64)]
 
 
 class dsm_hparams(ctypes.Structure):
@@ -135,8 +135,9 @@ def _stream(stream) -> c_void_p:
     return c_void_p(stream.cuda_stream)
 
 
-def make_layout(tensors):
-    """A dsm_layout from objects with numel, grad_scale, kind and wd; keep the result alive while used."""
+def make_layout(tensors, first_element: int = 0):
+    """A dsm_layout from objects with numel, grad_scale, kind and wd; keep the result alive while used.
+    first_element: the layout's first element within a larger model (a parameter shard), else 0."""
     arr = (dsm_tensor * len(tensors))()
     for i, t in enumerate(tensors):
         arr[i].numel = int(t.numel)
@@ -144,7 +145,7 @@ def make_layout(tensors):
         arr[i].kind = int(t.kind)
         arr[i].wd = int(getattr(t, "wd", 1))
         arr[i].reserved = 0
-    lay = dsm_layout(ctypes.cast(arr, POINTER(dsm_tensor)), len(tensors))
+    lay = dsm_layout(ctypes.cast(arr, POINTER(dsm_tensor)), len(tensors), int(first_element))
     lay._keep = arr
     return lay
 
@@ -296,14 +297,15 @@ class DistributedSignMomentum:
 
     tensors: objects with numel, grad_scale, kind, wd; hp: an object with
     the dsm_hparams field names.  x0: optional float32 torch tensor of d
-    elements (host or device).
+    elements (host or device).  first_element: where this layout starts in a
+    larger model of which it is a parameter shard (dsm_layout.first_element).
     """
 
     shapes = None   # the tensors' shapes, for a problem built by from_tensors
 
-    def __init__(self, tensors, n: int, tau: int, hp, device="cuda", x0=None, stream=None):
+    def __init__(self, tensors, n: int, tau: int, hp, device="cuda", x0=None, stream=None, first_element: int = 0):
         import torch
-        self.layout = make_layout(tensors)
+        self.layout = make_layout(tensors, first_element)
         self.hp = make_hparams(hp)
         self.n, self.tau = int(n), int(tau)
         self.nbytes = dsm_state_bytes(self.layout, self.n, self.hp)

@@ -30,7 +30,7 @@ int main(int argc, char** argv) {
         {2048, 1e-3f, DSM_KIND_LN_W, 1, 0},
     };
     const uint32_t count = 3;
-    const dsm_layout layout = {tensors, count};
+    const dsm_layout layout = {tensors, count, 0};  /* a whole model: first_element 0 */
     dsm_hparams hp;
     uint32_t n, tau;
     int rounds;

@@ -39,6 +39,20 @@ def test_struct_sizes_match_header_layout():
     assert ctypes.sizeof(dsm.dsm_tensor) == 24
     assert ctypes.sizeof(dsm.dsm_hparams) == 80
     assert ctypes.sizeof(dsm.dsm_tensor_stats) == 48
+    assert ctypes.sizeof(dsm.dsm_layout) == 24
+    assert dsm.dsm_layout.first_element.offset == 16
+
+
+def test_first_element_must_be_a_multiple_of_4(lib):
+    """A parameter shard starts at a multiple of 4 elements of the larger model (the synthetic draws come in
+    pairs and the randomized sign's Philox blocks in fours)."""
+    tensors = W.gpt2_layout(2, 64, 256)
+    hp = dsm.make_hparams(W.HParams())
+    assert dsm.dsm_state_bytes(dsm.make_layout(tensors, 1 << 20), 4, hp) > 0
+    for bad in (2, 6, 1 << 61):
+        with pytest.raises(dsm.DsmError) as e:
+            dsm.dsm_state_bytes(dsm.make_layout(tensors, bad), 4, hp)
+        assert "first_element" in str(e.value)
 
 
 def _args(tensors=None, n=4, hp=None):

@@ -207,3 +207,17 @@ def test_threads_do_not_change_results():
 def test_outside_element_is_refused():
     with pytest.raises(ValueError):
         C.CxxOracleRun(W.flat_layout(10, 1.0), 2, 1, ADAMW, elems=np.array([0, 10]))
+
+
+@pytest.mark.parametrize("first_element", [64, (1 << 35) + 8, (1 << 59) + 4096])
+def test_first_element_equals_numpy_oracle(first_element):
+    """A layout placed far into a larger model (64-bit draw indices, Philox counters above 2^32)."""
+    hp = dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, grad_dtype=W.BF16)
+    o = O.OracleRun(RAGGED, 3, 2, hp, with_stats=True, first_element=first_element)
+    c = C.CxxOracleRun(RAGGED, 3, 2, hp, with_stats=True, first_element=first_element)
+    _compare(c, o, "init")
+    for t in range(2):
+        o.run_round()
+        c.run_round()
+        _compare(c, o, t)
+        assert c.last_stats == o.last_stats
