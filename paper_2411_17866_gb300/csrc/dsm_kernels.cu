@@ -163,7 +163,7 @@ __device__ __forceinline__ void global_elem_generic(const Problem& p, const Glob
     const float x0 = x;
     float r = 0.f;
     if (MODE == 0 && g.sign_mode != 0)
-        r = philox_unit(word_of(philox_block(gi >> 2, g.philox_k0, g.philox_k1), gi & 3));
+        r = philox_unit(word_of(philox_block((gi >> 2) + g.philox_q0, g.philox_k0, g.philox_k1), gi & 3));
     float acc = 0.f;
     for (uint32_t i = 0; i < p.n; ++i) acc = __fadd_rn(acc, __fsub_rn(x0, p.X[i * p.d_stride + gi]));
     const float D = __fdiv_rn(acc, g.n_f);
@@ -221,7 +221,7 @@ __device__ __forceinline__ void global_vec_generic(const Problem& p, const Globa
     }
     float ru[4] = {0.f, 0.f, 0.f, 0.f};
     if (MODE == 0 && g.sign_mode != 0) {
-        const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+        const uint4 b = philox_block((gi >> 2) + g.philox_q0, g.philox_k0, g.philox_k1);
         ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
     }
     float D[4], xn[4], dr[4] = {0.f, 0.f, 0.f, 0.f};
@@ -326,7 +326,7 @@ __global__ void __launch_bounds__(kThreads) k_global(Problem p, GlobalScalars g)
             const uint64_t gi = td.start + e0;  // a multiple of 4: the four words of one Philox block
             float ru[4] = {0.f, 0.f, 0.f, 0.f};
             if (MODE == 0 && g.sign_mode != 0) {
-                const uint4 b = philox_block(gi >> 2, g.philox_k0, g.philox_k1);
+                const uint4 b = philox_block((gi >> 2) + g.philox_q0, g.philox_k0, g.philox_k1);
                 ru[0] = philox_unit(b.x); ru[1] = philox_unit(b.y); ru[2] = philox_unit(b.z); ru[3] = philox_unit(b.w);
             }
 #pragma unroll
@@ -366,29 +366,47 @@ __global__ void __launch_bounds__(kThreads) k_stats(Problem p, uint32_t producer
     unsigned long long c0 = 0, c1 = 0, c2 = 0, c3 = 0;
     const uint32_t first =
         td.tile_end - td.tile_begin > producer_grid ? td.tile_end - producer_grid : td.tile_begin;
-    for (uint32_t t = first + threadIdx.x; t < td.tile_end; t += blockDim.x) {
-        const StatPartial q = p.partials[t];
-        a += q.delta_sq; b += q.drift;
-        c0 += q.zero_sign; c1 += q.flips; c2 += q.unanimous; c3 += q.clamped;
-    }
-    __shared__ double s_d[kThreads][2];
-    __shared__ unsigned long long s_c[kThreads][4];
-    s_d[threadIdx.x][0] = a; s_d[threadIdx.x][1] = b;
-    s_c[threadIdx.x][0] = c0; s_c[threadIdx.x][1] = c1; s_c[threadIdx.x][2] = c2; s_c[threadIdx.x][3] = c3;
-    __syncthreads();
-    for (uint32_t off = kThreads / 2; off > 0; off >>= 1) {
-        if (threadIdx.x < off) {
-            s_d[threadIdx.x][0] += s_d[threadIdx.x + off][0];
-            s_d[threadIdx.x][1] += s_d[threadIdx.x + off][1];
+    // each thread sums partials first + tid, first + tid + 256, ...; the loads of up to 4 of them are
+    // issued before their additions (a tensor has at most producer_grid partials)
+    for (uint32_t t0 = first + threadIdx.x; t0 < td.tile_end; t0 += 4 * kThreads) {
+        StatPartial q[4];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) s_c[threadIdx.x][k] += s_c[threadIdx.x + off][k];
+        for (int u = 0; u < 4; ++u)
+            if (t0 + u * kThreads < td.tile_end) q[u] = p.partials[t0 + u * kThreads];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (t0 + u * kThreads < td.tile_end) {
+                a += q[u].delta_sq; b += q[u].drift;
+                c0 += q[u].zero_sign; c1 += q[u].flips; c2 += q[u].unanimous; c3 += q[u].clamped;
+            }
         }
-        __syncthreads();
     }
+    // the lanes of each warp by shuffles in a fixed pattern, then the warps in order
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        a += __shfl_down_sync(0xffffffffu, a, off);
+        b += __shfl_down_sync(0xffffffffu, b, off);
+        c0 += __shfl_down_sync(0xffffffffu, c0, off);
+        c1 += __shfl_down_sync(0xffffffffu, c1, off);
+        c2 += __shfl_down_sync(0xffffffffu, c2, off);
+        c3 += __shfl_down_sync(0xffffffffu, c3, off);
+    }
+    __shared__ double s_d[kThreads / 32][2];
+    __shared__ unsigned long long s_c[kThreads / 32][4];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        s_d[warp][0] = a; s_d[warp][1] = b;
+        s_c[warp][0] = c0; s_c[warp][1] = c1; s_c[warp][2] = c2; s_c[warp][3] = c3;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
         TensorStats o;
-        o.delta_sq = s_d[0][0]; o.drift = s_d[0][1];
-        o.zero_sign = s_c[0][0]; o.flips = s_c[0][1]; o.unanimous = s_c[0][2]; o.clamped = s_c[0][3];
+        o.delta_sq = 0.0; o.drift = 0.0;
+        o.zero_sign = o.flips = o.unanimous = o.clamped = 0;
+        for (int w = 0; w < kThreads / 32; ++w) {
+            o.delta_sq += s_d[w][0]; o.drift += s_d[w][1];
+            o.zero_sign += s_c[w][0]; o.flips += s_c[w][1]; o.unanimous += s_c[w][2]; o.clamped += s_c[w][3];
+        }
         p.stats[T] = o;
     }
 }

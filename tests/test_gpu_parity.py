@@ -124,6 +124,11 @@ FUSED = [
     ("sgdm-rsignpm-n3-t2", dataclasses.replace(SGDM, sign_mode=W.RSIGN_PM, grad_dtype=W.BF16), 3, 2),
     ("adamw-n1-t1", ADAMW, 1, 1),
     ("adamw-n5-t2", ADAMW, 5, 2),
+    # the split kernel (AdamW, 5 to 8 workers): odd and even worker counts, randomized signs, tau = 1
+    # (every fused launch after the first starts the workers from x)
+    ("adamw-f32-n6-t1-rsignpm", dataclasses.replace(ADAMW, sign_mode=W.RSIGN_PM, rsign_B=0.5, seed=4), 6, 1),
+    ("adamw-bf16-n7-t3-rsign0", dataclasses.replace(ADAMW, grad_dtype=W.BF16, sign_mode=W.RSIGN_ZERO,
+                                                     rsign_B=1.0), 7, 3),
     ("adamw-n9-deferred-reset", ADAMW, 9, 2),
     ("sgdm-rsign-n16-deferred-reset", SGDM, 16, 1),
     ("slowmo-unfused", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO), 4, 2),
@@ -292,6 +297,54 @@ def test_statistics_of_the_hand_built_global_step():
     for key in ("zero_sign", "flips", "unanimous", "clamped"):
         assert st[key] == want["stats"][key], key
     run.close()
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["unfused", "fused"])
+def test_parameter_shards_of_one_model(fused):
+    """One model cut into three parameter shards (paper_2411_17866_gb300/shard.py), each run by the
+    library with its pieces as the layout and its first_element, one after another on this GPU: every shard
+    equals the whole-model oracle on its range bit for bit over two rounds (randomized sign, bf16
+    gradients), and the shards' per-piece statistics summed per tensor equal the whole-model statistics."""
+    from paper_2411_17866_gb300 import shard as S
+    model = RAGGED
+    n, tau, world = 3, 2, 3
+    hp = dataclasses.replace(ADAMW, sign_mode=W.RSIGN_PM, rsign_B=0.5, grad_dtype=W.BF16, seed=9,
+                             flags=W.FLAG_FUSED_ROUND if fused else 0)
+    whole = O.OracleRun(model, n, tau, hp, with_stats=True)
+    whole_stats = []
+    for _ in range(2):
+        whole.run_round()
+        whole_stats.append(whole.last_stats)
+    per_round = [[], []]
+    for r in range(world):
+        sh = S.shard_layout(model, world, r)
+        run = dsm.DistributedSignMomentum(sh.tensors, n, tau, hp, first_element=sh.first_element)
+        ora = O.OracleRun(model, n, tau, hp, elems=np.arange(sh.first_element, sh.first_element + sh.count))
+        for t in range(2):
+            st = run.synthetic_round(with_stats=True)
+            ora.run_round()
+            compare_state(run, ora)
+            per_round[t].append(S.stats_by_tensor(sh, st, len(model)))
+        run.close()
+    for t in range(2):
+        compare_stats(S.reduce_stats(per_round[t]), whole_stats[t], n)
+
+
+@pytest.mark.parametrize("first_element", [1 << 20, (1 << 35) + 8, (1 << 59) + 4096],
+                         ids=["2^20", "2^35+8", "2^59+4096"])
+def test_first_element_far_into_a_larger_model(first_element):
+    """A layout placed far into a larger model: the 64-bit key offsets of the synthetic draws and the
+    Philox counter's high word (first_element/4 >= 2^32) against the oracle with the same first_element."""
+    hp = dataclasses.replace(SGDM, sign_mode=W.RSIGN_ZERO, rsign_B=1e-2, grad_dtype=W.BF16)
+    for h in (hp, dataclasses.replace(ADAMW, flags=W.FLAG_FUSED_ROUND)):
+        run = dsm.DistributedSignMomentum(RAGGED, 4, 2, h, first_element=first_element)
+        ora = O.OracleRun(RAGGED, 4, 2, h, first_element=first_element, with_stats=True)
+        for _ in range(2):
+            st = run.synthetic_round(with_stats=True)
+            ora.run_round()
+            compare_state(run, ora)
+            compare_stats(st, ora.last_stats, 4)
+        run.close()
 
 
 def test_x0_from_device_and_host():
@@ -529,6 +582,8 @@ RESET = [
     ("sgdm-rsign-n8-t2", SGDM, 8, 2),
     ("sgdm-bf16-n2-t1", dataclasses.replace(SGDM, grad_dtype=W.BF16, sign_mode=W.SIGN), 2, 1),
     ("adamw-n9-generic-t2", ADAMW, 9, 2),
+    ("adamw-bf16-n8-t1", dataclasses.replace(ADAMW, grad_dtype=W.BF16), 8, 1),
+    ("adamw-n7-t2", ADAMW, 7, 2),
     ("slowmo-adamw-n4-t2", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_SLOWMO, g_b1=0.5, g_eta=0.8), 4, 2),
     ("global-adamw-n3-t2", dataclasses.replace(ADAMW, global_mode=W.GLOBAL_ADAMW), 3, 2),
 ]

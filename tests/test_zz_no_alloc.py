@@ -57,8 +57,9 @@ def _caller_buffers(run, n):
     return x, m, reps
 
 
-def _noalloc(tensors, n, hp, gamma, round_, x, m, reps, stride, stats=None, stats_is_device=False):
-    dsm.dsm_global_step_noalloc(dsm.make_layout(tensors), n, dsm.make_hparams(hp), gamma, round_, x.data_ptr(),
+def _noalloc(tensors, n, hp, gamma, round_, x, m, reps, stride, stats=None, stats_is_device=False, first_element=0):
+    dsm.dsm_global_step_noalloc(dsm.make_layout(tensors, first_element), n, dsm.make_hparams(hp), gamma, round_,
+                                x.data_ptr(),
                                 m.data_ptr(), reps.data_ptr(), stride,
                                 stats if not stats_is_device else stats.data_ptr(), stats_is_device=stats_is_device)
 
@@ -114,12 +115,14 @@ def test_noalloc_global_step_matches_handle_path(name, hp, n, tau):
     run.close()
 
 
+@pytest.mark.parametrize("first_element", [0, (1 << 35) + 8], ids=["whole-model", "shard-at-2^35"])
 @pytest.mark.parametrize("name,hp,n,tau", CASES, ids=[c[0] for c in CASES])
-def test_noalloc_global_step_matches_oracle(name, hp, n, tau):
+def test_noalloc_global_step_matches_oracle(name, hp, n, tau, first_element):
     """Two rounds: the oracle's local steps, then its state uploaded to the caller's buffers and the global
-    step run by dsm_global_step_noalloc; x, m and every replica bit for bit, statistics to tolerance."""
+    step run by dsm_global_step_noalloc; x, m and every replica bit for bit, statistics to tolerance.  A layout
+    placed far into a larger model moves the randomized sign's Philox counter."""
     _need_gpu()
-    ora = O.OracleRun(LAYOUT, n, tau, hp, with_stats=True)
+    ora = O.OracleRun(LAYOUT, n, tau, hp, with_stats=True, first_element=first_element)
     d = ora.d
     stride = (d + 63) // 64 * 64
     for t in range(2):
@@ -131,7 +134,7 @@ def test_noalloc_global_step_matches_oracle(name, hp, n, tau):
         for i in range(n):
             reps[i * stride:i * stride + d] = torch.from_numpy(ora.X[i])
         host_stats = (dsm.dsm_tensor_stats * len(LAYOUT))()
-        _noalloc(LAYOUT, n, hp, ora.gamma, ora.t, x, m, reps, stride, host_stats)
+        _noalloc(LAYOUT, n, hp, ora.gamma, ora.t, x, m, reps, stride, host_stats, first_element=first_element)
         ora.global_step()
         torch.cuda.synchronize()
         assert_bitexact(x.cpu().numpy(), ora.x, f"x, round {t}")
