@@ -479,6 +479,32 @@ def kernel_figures(wl, res, peak):
     return out
 
 
+def copy_gbs(nbytes, dev, stream, reps=8):
+    """Bandwidth of a plain device-to-device copy that moves `nbytes` (half read, half written; capped at
+    2 GiB), over its CUDA-event time (median of `reps`), with L2 flushed before each copy: the copy roofline
+    at a launch of that size, which small launches (ramp and tail of a short kernel) keep below the large
+    copy's peak."""
+    import torch
+    nbytes = min(int(nbytes), 2 << 30)
+    src = torch.empty(max(nbytes // 8, 1), dtype=torch.float32, device=dev)
+    dst = torch.empty_like(src)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # larger than the 129 MB L2
+    times = []
+    for r in range(reps + 2):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        dst.copy_(src)
+        b.record(stream)
+        torch.cuda.synchronize()
+        if r >= 2:
+            times.append(a.elapsed_time(b) / 1e3)
+    moved = 2 * src.numel() * 4
+    del src, dst, flush
+    return moved / statistics.median(times) / 1e9
+
+
 def workload_sweep(dev, stream, peak, skip, steps=3, warmup=2):
     """Every measured workload (fused round, as configured) timed briefly in this process with CUDA events:
     params/s of the round and each kernel's fraction of both peaks.  `skip` maps a workload already timed
@@ -499,6 +525,13 @@ def workload_sweep(dev, stream, peak, skip, steps=3, warmup=2):
         del run
         torch.cuda.empty_cache()
         out[key] = sweep_entry(wl, res, peak, steps)
+    for key, e in out.items():   # the plain copy's bandwidth at each workload's local-step launch size
+        wl = W.WORKLOADS[key]
+        c = copy_gbs(local_step_bytes(wl), dev, stream)
+        e["copy_gbs_at_launch_size"] = c
+        if "local_step_gbs" in e:
+            e["local_step_frac_of_copy_at_launch_size"] = e["local_step_gbs"] / c
+        torch.cuda.empty_cache()
     return out
 
 
@@ -640,8 +673,9 @@ def main():
         sweep = workload_sweep(dev, stream, peak, done)
         line["workloads"] = {"note": "each workload's fused round as configured, timed in this job with CUDA "
                                      "events (2 untimed + 3 timed rounds; the bench workload's entry is the "
-                                     "timed region above); fractions of the measured copy peak and of 8 TB/s; "
-                                     "flat1m's launches (50-117 MB) fit in L2",
+                                     "timed region above); fractions of the measured copy peak and of 8 TB/s, "
+                                     "and of a plain copy moving one local-step launch's bytes (at most 2 GiB, "
+                                     "L2 flushed before each copy)",
                              "clocks": sampler.stop() if sampler else None, **sweep}
     if not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(wl)
