@@ -41,7 +41,10 @@ Parity pins: each function here is pinned by a test in
 ``tests/test_oracle_pins.py`` against something other than itself (the
 exact worked example, closed forms, library routines, published test
 vectors, invariants, Lemma 1).  The per-tensor statistics have no printed
-values in the paper; they are pinned by invariants and by numpy reductions.
+values in the paper; they are pinned by hand-computed values of two d = 8
+global steps (tests/golden/worked_example_d8.json, stats_example_d8.json),
+by invariants and by numpy reductions.  The C++ oracle (dsm_oracle.cpp)
+computes the same values bit for bit.
 """
 from __future__ import annotations
 
