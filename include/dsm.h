@@ -244,8 +244,18 @@ int dsm_set_gamma(dsm_handle* h, float gamma);
  *   g_i[e] = s_T*(u(seed,0,step,e) - 1/2) + fp32(0.1f*s_T)*(u(seed,1,i,e) - 1/2)
  * with u the top 24 bits of a SplitMix64 output scaled by 2^-24, rounded to
  * bf16 (nearest even) when grad_dtype is DSM_BF16.  Stands in for the
- * backward pass.  Asynchronous. */
+ * backward pass.  Worker i draws with index first_worker + i (0 unless
+ * dsm_set_first_worker set it).  Asynchronous. */
 int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream);
+
+/* Place the handle's n workers at positions first_worker .. first_worker+n-1
+ * of a larger set of Algorithm 1's workers: a process that holds one
+ * contiguous group of the workers of a worker-sharded deployment (the
+ * paper's workers are devices, Sec. 5).  Worker i then draws the synthetic
+ * gradient of worker first_worker + i in dsm_fill_synthetic_grads; nothing
+ * else depends on it.  Any time; takes effect at the next fill.  DSM_EINVAL
+ * for a NULL handle, DSM_ERANGE if first_worker + n exceeds 2^32. */
+int dsm_set_first_worker(dsm_handle* h, uint32_t first_worker);
 
 /* Device pointer to worker `worker`'s gradient buffer, for a caller that
  * writes the update directions' inputs itself (the stochastic gradients
@@ -356,6 +366,24 @@ int dsm_cosine_gamma(float peak, float final_ratio, uint64_t warmup_steps, uint6
  * with DSM_FLAG_RESET_LOCAL_STATE) and the global AdamW count t + 1.  Only
  * between rounds, else DSM_ESTATE. */
 int dsm_set_round(dsm_handle* h, uint64_t round);
+
+/* End round t of Algorithm 1 with a global model computed elsewhere.  In a
+ * worker-sharded deployment the processes that own the model's parameter
+ * ranges compute x_{t+1,0} = x_{t,0} - eta*gamma_t*(S(u_{t+1}) + lambda*x_{t,0})
+ * (Eq. (model-update)) and the global momentum, from every worker's model,
+ * so the handles that hold the workers do not run dsm_global_step: each
+ * ends its round with this call instead.  Needs all tau local steps of the
+ * round (DSM_ESTATE otherwise); a last local step deferred by
+ * DSM_FLAG_FUSED_ROUND runs first, so that the workers' base-optimizer
+ * states are complete.  Then x <- x_next (d fp32 values, in host or device
+ * memory, x_is_device), every worker restarts from x (Algorithm 1's
+ * synchronisation; the next local step reads x, as after a fused round),
+ * t <- t + 1 (the randomized sign's key and the global AdamW count advance
+ * as after dsm_global_step) and, with DSM_FLAG_RESET_LOCAL_STATE, the
+ * base optimizer restarts.  The handle's own m (and global v) are left as
+ * they are.  With host memory the call synchronises the stream.
+ * DSM_EINVAL for NULL arguments. */
+int dsm_end_round(dsm_handle* h, const float* x_next, int x_is_device, dsm_stream_t stream);
 
 /* Describe the handle (sizes, t and k of Algorithm 1, gamma_t) into *out.
  * Host only.  DSM_EINVAL for NULL arguments. */

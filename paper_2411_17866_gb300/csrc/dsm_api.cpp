@@ -218,6 +218,7 @@ struct dsm_handle {
     SgdmScalars pending_sa{};
     uint64_t j = 0;        // AdamW step count of the last local step (restarts each round with the reset flag)
     uint64_t first_element = 0;  // the layout's first element within a larger model (a parameter shard)
+    uint32_t first_worker = 0;   // worker 0's index in a larger set of workers (synthetic gradients)
     // local steps with host gradients (dsm_local_step_host_grads): chunk c covers tiles
     // [chunk_tile[c], chunk_tile[c+1]); ev_copied[c] marks its gradients in the arena
     std::vector<uint32_t> chunk_tile;
@@ -541,13 +542,21 @@ int dsm_fill_synthetic_grads(dsm_handle* h, uint64_t step, dsm_stream_t stream) 
     GradKeys k;
     k.step = shard_key(draw_key(h->hp.seed, 0, step), h->first_element);
     for (uint32_t i = 0; i < kMaxWorkers; ++i)
-        k.worker[i] = i < h->n ? shard_key(draw_key(h->hp.seed, 1, i), h->first_element) : 0;
+        k.worker[i] = i < h->n ? shard_key(draw_key(h->hp.seed, 1, uint64_t(h->first_worker) + i), h->first_element) : 0;
     DeviceGuard guard(h->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     int rc = materialize_pending(h, S(stream));
     if (rc != DSM_OK) return rc;
     cudaError_t err = launch_grad_fill(h->prob, h->shape, k, S(stream));
     if (err != cudaSuccess) return cuda_fail(err, "launch grad fill");
+    return DSM_OK;
+}
+
+int dsm_set_first_worker(dsm_handle* h, uint32_t first_worker) {
+    if (!h) return fail(DSM_EINVAL, "handle is NULL");
+    if (uint64_t(first_worker) + h->n > (uint64_t(1) << 32))
+        return fail(DSM_ERANGE, "workers %u .. %u + %u exceed 2^32", first_worker, first_worker, h->n);
+    h->first_worker = first_worker;
     return DSM_OK;
 }
 
@@ -822,6 +831,29 @@ int dsm_set_round(dsm_handle* h, uint64_t round) {
     }
     h->gb1_pow = q1;
     h->gb2_pow = q2;
+    return DSM_OK;
+}
+
+int dsm_end_round(dsm_handle* h, const float* x_next, int x_is_device, dsm_stream_t stream) {
+    if (!h || !x_next) return fail(DSM_EINVAL, "NULL argument");
+    if (h->k != h->tau)
+        return fail(DSM_ESTATE, "ending round %llu needs its %u local steps, %u done", (unsigned long long)h->t,
+                    h->tau, h->k);
+    DeviceGuard guard(h->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    cudaStream_t s = S(stream);
+    int rc = materialize_pending(h, s);  // the workers' last base-optimizer step
+    if (rc != DSM_OK) return rc;
+    cudaError_t err = cudaMemcpyAsync(h->prob.x, x_next, size_t(h->al.d) * 4, copy_kind(x_is_device, true), s);
+    if (err != cudaSuccess) return cuda_fail(err, "write the next global model");
+    h->replicas_stale = true;  // every worker restarts from x
+    h->t += 1;
+    h->k = 0;
+    h->gb1_pow *= double(h->hp.g_b1);
+    h->gb2_pow *= double(h->hp.g_b2);
+    begin_next_round_states(h);
+    if (!x_is_device && (err = cudaStreamSynchronize(s)) != cudaSuccess)
+        return cuda_fail(err, "synchronise after writing the global model");
     return DSM_OK;
 }
 

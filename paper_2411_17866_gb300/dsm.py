@@ -86,6 +86,8 @@ _PROTOS = {
     "dsm_read_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
     "dsm_write_params": (c_int, [c_void_p, c_int, c_uint32, c_void_p, c_uint64, c_uint64, c_int, c_void_p]),
     "dsm_set_round": (c_int, [c_void_p, c_uint64]),
+    "dsm_set_first_worker": (c_int, [c_void_p, c_uint32]),
+    "dsm_end_round": (c_int, [c_void_p, c_void_p, c_int, c_void_p]),
     "dsm_cosine_gamma": (c_int, [c_float, c_float, c_uint64, c_uint64, c_uint64, POINTER(c_float)]),
     "dsm_get_info": (c_int, [c_void_p, POINTER(dsm_info)]),
     "dsm_check_guards": (c_int, [c_void_p, c_void_p, POINTER(c_uint32)]),
@@ -249,6 +251,15 @@ def dsm_set_round(h, round_: int) -> None:
     _check(load_library().dsm_set_round(h, round_), "dsm_set_round")
 
 
+def dsm_set_first_worker(h, first_worker: int) -> None:
+    _check(load_library().dsm_set_first_worker(h, first_worker), "dsm_set_first_worker")
+
+
+def dsm_end_round(h, x_ptr: int, x_is_device: bool, stream=None) -> None:
+    _check(load_library().dsm_end_round(h, c_void_p(x_ptr), int(bool(x_is_device)), _stream(stream)),
+           "dsm_end_round")
+
+
 def dsm_cosine_gamma(peak: float, final_ratio: float, warmup_steps: int, total_steps: int, step: int) -> float:
     out = c_float()
     _check(load_library().dsm_cosine_gamma(peak, final_ratio, warmup_steps, total_steps, step, byref(out)),
@@ -364,6 +375,10 @@ class DistributedSignMomentum:
     def fill_synthetic_grads(self, step, stream=None):
         dsm_fill_synthetic_grads(self.h, step, stream)
 
+    def set_first_worker(self, first_worker):
+        """Worker i draws the synthetic gradients of worker first_worker + i of a larger set."""
+        dsm_set_first_worker(self.h, first_worker)
+
     def load_grads(self, src, stream=None):
         dsm_load_grads(self.h, src.data_ptr(), src.is_cuda, stream)
 
@@ -408,6 +423,15 @@ class DistributedSignMomentum:
         arr = (dsm_tensor_stats * self.num_tensors)()
         dsm_global_step(self.h, stream, arr)
         return [a.as_dict() for a in arr]
+
+    def end_round(self, x_next, stream=None):
+        """End the round with a global model computed elsewhere (d fp32 values, CPU or CUDA tensor):
+        every worker restarts from it and the round counter advances; no global step runs here."""
+        import torch
+        x_next = x_next.contiguous()
+        if x_next.dtype != torch.float32 or x_next.numel() != self.d:
+            raise ValueError(f"x_next must hold {self.d} float32 values")
+        dsm_end_round(self.h, x_next.data_ptr(), x_next.is_cuda, stream)
 
     def synthetic_round(self, stream=None, with_stats=False):
         """tau x (synthetic gradients + local step), then the global step."""

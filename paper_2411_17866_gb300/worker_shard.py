@@ -33,6 +33,8 @@ The compute backend is an object with
                                     ([n, count] tensor); returns the range's new x and the statistics of
                                     the shard's pieces (or None);
   restart(x)                        the new global model x (all d values): every worker starts from it.
+Two backends exist: the oracle's (tests/test_worker_shard.py) and LibraryWorkers below, which runs the
+rank's workers and the owner's global step in the library on the process's GPU.
 This module holds no arithmetic of the method; it places the workers and the ranges, and moves data.
 """
 from __future__ import annotations
@@ -113,3 +115,72 @@ class WorkerShardedRound:
             return None
         mine = S.stats_by_tensor(self.shard, piece_stats, len(self.tensors))
         return S.all_reduce_stats(mine)
+
+
+class LibraryWorkers:
+    """The compute backend on this process's CUDA device, through the library's C ABI.
+
+    - The rank's workers are one handle of group.count workers over the whole model, placed at
+      group.first_worker (dsm_set_first_worker), so that they draw the synthetic gradients of those
+      workers of the n.
+    - The owned range's global step is dsm_global_step_noalloc on the owner's x and m of the range and
+      the n models of the range (Algorithm 1's global step, the one that entry point runs), with the
+      range's layout placed at its first element (dsm_layout.first_element: the randomized sign's
+      counters are those of the whole model).
+    - The restart is dsm_end_round with the gathered x: the handle's workers start the next round from
+      it, their base-optimizer states carry over.
+    comm_device: where the collectives' tensors live ("cpu" for gloo, the CUDA device for NCCL)."""
+
+    def __init__(self, tensors, n: int, tau: int, hp, group: WorkerGroup, shard: S.Shard, device="cuda",
+                 comm_device="cpu"):
+        import torch
+        from . import dsm
+        self._dsm = dsm
+        self.tau, self.n = tau, n
+        self.device = torch.device(device)
+        self.comm = torch.device(comm_device)
+        self.run = dsm.DistributedSignMomentum(tensors, group.count, tau, hp, device=self.device)
+        self.run.set_first_worker(group.first_worker)
+        self.shard = shard
+        self.layout = dsm.make_layout(shard.tensors, first_element=shard.first_element)
+        self.hparams = dsm.make_hparams(hp)
+        # the owner's state of its range: x, m (m_0 = 0) and the n models, rows padded to a multiple of 8
+        self.stride = max(8, -(-shard.count // 8) * 8)
+        self.m = torch.zeros(max(shard.count, 1), dtype=torch.float32, device=self.device)
+        self.x = torch.empty(max(shard.count, 1), dtype=torch.float32, device=self.device)
+        self.X = torch.empty((n, self.stride), dtype=torch.float32, device=self.device)
+
+    def local_steps(self, t):
+        for k in range(self.tau):
+            self.run.fill_synthetic_grads(t * self.tau + k)
+            self.run.local_step()
+
+    def replicas(self):
+        import torch
+        if self.comm.type == "cuda":
+            return torch.stack([self.run.replica_view(i) for i in range(self.run.n)])
+        return torch.stack([self.run.read(self._dsm.BUF_REPLICA, i) for i in range(self.run.n)])
+
+    def global_step(self, shard, X_shard, t):
+        import torch
+        dsm = self._dsm
+        count = shard.count
+        if count == 0:
+            return torch.empty(0, dtype=torch.float32, device=self.comm), []
+        with torch.cuda.device(self.device):
+            self.X[:, :count].copy_(X_shard.to(self.device))
+            self.run.read(dsm.BUF_X, offset=shard.first_element, count=count, out=self.x[:count])
+            stats = (dsm.dsm_tensor_stats * len(shard.pieces))()
+            dsm.dsm_global_step_noalloc(self.layout, self.n, self.hparams, self.run.info().gamma, t,
+                                        self.x.data_ptr(), self.m.data_ptr(), self.X.data_ptr(), self.stride,
+                                        stats)
+            return self.x[:count].to(self.comm), [s.as_dict() for s in stats]
+
+    def restart(self, x):
+        import torch
+        with torch.cuda.device(self.device):
+            self.run.end_round(x)
+
+    def momentum(self):
+        """The owner's global momentum of its range (CPU)."""
+        return self.m[:self.shard.count].cpu()

@@ -144,6 +144,8 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert lib.dsm_set_gamma(None, ctypes.c_float(1.0)) == dsm.DSM_EINVAL
     assert lib.dsm_fill_synthetic_grads(None, 0, None) == dsm.DSM_EINVAL
     assert lib.dsm_read_params(None, 0, 0, None, 0, 0, 0, None) == dsm.DSM_EINVAL
+    assert lib.dsm_set_first_worker(None, 0) == dsm.DSM_EINVAL
+    assert lib.dsm_end_round(None, None, 0, None) == dsm.DSM_EINVAL
     assert lib.dsm_destroy(None) == dsm.DSM_OK
 
 
