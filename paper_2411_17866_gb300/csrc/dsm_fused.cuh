@@ -34,24 +34,32 @@ namespace {
 // A CTA walks its tiles worker by worker; each thread keeps the next
 // kFusedDepth (tile, worker) items in flight with cp.async into its own
 // shared-memory slots: x_i, m_i (v_i) and g_i per item, and x, m with a tile's
-// first worker into a slot pair kept per tile parity.
+// first worker into a set of slots for the tile.
 // Items in flight per thread: 2, or 3 for AdamW with more than 4 workers,
 // whose registers already limit the resident CTAs (measured on GB300: depth 2
 // gives 0.92 / 1.00 of the copy bandwidth on GPT-2 S (AdamW, n = 4) / L
 // (SGD-momentum, n = 8), depth 3 gives 0.85 on GPT-2 M (AdamW, n = 8) where
 // depth 2 gives 0.79).  Staging x and m once per tile instead of in every
 // item's slots (59 instead of 72 KB per CTA for GPT-2 M) raised GPT-2 M to
-// 0.87; four items in flight in the same 72 KB gave 0.86.
+// 0.87; four items in flight in the same 72 KB gave 0.86.  The x/m slots of
+// tile q are set q % S: two sets (by tile parity), or one for AdamW with more
+// than 4 workers (50 instead of 59 KB per CTA: GPT-2 M 0.88 against 0.87,
+// where one set for n = 4 gave 0.93 / 0.94 against 0.94 / 0.95 on GPT-2 XL / S).
 constexpr int kGlobalSign = 0, kGlobalRuntime = 1, kGlobalAdamW = 2;
 __host__ __device__ constexpr int fused_depth(bool adamw, int nw) { return (adamw && nw > 4) ? 3 : 2; }
+// Sets of x/m slots S.  A tile's set is refilled with the first item of the
+// tile S tiles later, issued when the item `depth` places before that one is
+// consumed; that item comes after the tile's own first item (which takes x
+// and m into registers) only if depth <= S * nw.
+__host__ __device__ constexpr int fused_glob_sets(bool adamw, int nw) { return (adamw && nw > 4) ? 1 : 2; }
 // Staging per thread: for every item in flight the worker's x_i, m_i (and v_i
 // for AdamW) in 16-byte slots and its gradient in an 8- or 16-byte slot; for
-// each of two tiles (by parity) x and m (and the global v) of the tile.
+// each set, x and m (and the global v) of a tile.
 __host__ __device__ constexpr int fused_states(bool adamw) { return adamw ? 3 : 2; }
 __host__ __device__ constexpr int fused_globals(int global) { return global == kGlobalAdamW ? 3 : 2; }
 __host__ __device__ constexpr size_t fused_smem(bool adamw, bool bf16, int nw, int global) {
     return (size_t(fused_depth(adamw, nw)) * (fused_states(adamw) * 16 + (bf16 ? 8 : 16)) +
-            2 * fused_globals(global) * 16) * kThreads;
+            size_t(fused_glob_sets(adamw, nw)) * fused_globals(global) * 16) * kThreads;
 }
 
 template <bool kAdamW, bool kBf16, int NW, int kGlobal>
@@ -60,10 +68,11 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
     constexpr int kFusedDepth = fused_depth(kAdamW, NW);
     constexpr int kStates = fused_states(kAdamW), kGlobals = fused_globals(kGlobal);
     constexpr int kGradBytes = kBf16 ? 8 : 16;
-    static_assert(kFusedDepth <= 2 * NW, "a tile's x and m slots are reused two tiles later");
+    constexpr int kGlobSets = fused_glob_sets(kAdamW, NW);
+    static_assert(kFusedDepth <= kGlobSets * NW, "a tile's x/m slots are refilled only after its first item");
     const bool from_global = opts & kFusedFromX, zero_state = opts & kFusedZeroState,
                keep_state = !(opts & kFusedDropState);
-    // [kFusedDepth][kStates][kThreads] float4 | [kFusedDepth][kThreads] gradients | [2][kGlobals][kThreads] float4
+    // [kFusedDepth][kStates][kThreads] float4 | [kFusedDepth][kThreads] gradients | [kGlobSets][kGlobals][kThreads] float4
     extern __shared__ float4 fsm[];
     char* const grad_base = reinterpret_cast<char*>(fsm + size_t(kFusedDepth) * kStates * kThreads);
     float4* const glob_base = reinterpret_cast<float4*>(grad_base + size_t(kFusedDepth) * kThreads * kGradBytes);
@@ -75,7 +84,7 @@ __global__ void __launch_bounds__(kThreads) k_fused_last_global(Problem p, AdamS
         return grad_base + (size_t(it % kFusedDepth) * kThreads + threadIdx.x) * kGradBytes;
     };
     auto glob_slot = [&](uint32_t q, int s) -> float4* {
-        return glob_base + (size_t(q & 1) * kGlobals + s) * kThreads + threadIdx.x;
+        return glob_base + (size_t(q % kGlobSets) * kGlobals + s) * kThreads + threadIdx.x;
     };
     // Issue item `it` (tile number it / NW of this CTA, worker it % NW); always commits one group.
     auto issue = [&](uint32_t it) {
