@@ -35,6 +35,7 @@ CASES = {
                                               seed=5),
     "adamw-fused-sign": dataclasses.replace(W.HParams(), flags=W.FLAG_FUSED_ROUND, seed=9),
     "sgdm-rsign0": dataclasses.replace(W.SGDM_HP, seed=2),
+    "adamw-reset-local": dataclasses.replace(W.HParams(), flags=W.FLAG_RESET_LOCAL_STATE, seed=4),
 }
 
 
@@ -66,7 +67,7 @@ def test_first_worker_draws_those_workers_gradients(dsm):
         run.close()
 
 
-@pytest.mark.parametrize("case", ["adamw-bf16-rsignpm", "adamw-fused-sign", "sgdm-rsign0"])
+@pytest.mark.parametrize("case", ["adamw-bf16-rsignpm", "adamw-fused-sign", "sgdm-rsign0", "adamw-reset-local"])
 def test_end_round_restarts_from_the_given_model(dsm, case):
     """dsm_end_round after the local steps leaves the handle where a handle that ran the global step itself
     is (x, replicas, base-optimizer states, round counter), and the next round's local steps agree."""
