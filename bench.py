@@ -152,6 +152,24 @@ def max_over_ranks(seconds: float, world: int) -> float:
     return float(t.item())
 
 
+# A timed region whose clocks show one of these reasons, or SM clocks well below their maximum with no
+# reason given (a clock lock left by someone else), is measured again once.
+REJECTED_CLOCK_REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
+
+
+def clocks_rejected(clocks) -> bool:
+    if not clocks:
+        return False
+    if set(REJECTED_CLOCK_REASONS) & set(clocks["reasons"]):
+        return True
+    return not clocks["reasons"] and clocks["sm_mhz"] < 0.9 * clocks["sm_max_mhz"]
+
+
+def any_rank(flag: bool, world: int) -> bool:
+    """True on every rank if any rank's flag is true (host-side gloo reduction)."""
+    return max_over_ranks(1.0 if flag else 0.0, world) > 0.5
+
+
 def rank_shard(wl, world: int, rank: int):
     """Rank r's part of the weak-scaling model: `world` copies of the workload's tensor list, cut into
     `world` contiguous shards of d parameters (shard r is copy r and starts at element r*d of that model).
@@ -588,6 +606,12 @@ def main():
 
     sampler = ClockSampler(local) if (rank == 0 and not args.no_clocks) else None
     t, res = time_rounds(run, wl, stream, 0, args.warmup, args.steps, world, sampler)
+    if any_rank(clocks_rejected(res["clocks"]), world):   # throttled or clock-locked: measure once more
+        first = res["clocks"]
+        sampler = ClockSampler(local) if (rank == 0 and not args.no_clocks) else None
+        t, res = time_rounds(run, wl, stream, t, 1, args.steps, world, sampler)
+        if res["clocks"] is not None and first is not None:
+            res["clocks"]["remeasured_after"] = {k: first[k] for k in ("sm_mhz", "reasons")}
     elapsed, clocks, fused, lazy = res["elapsed"], res["clocks"], res["fused"], res["lazy"]
 
     # end to end through the C ABI with host buffers: per round, tau x (pinned host -> device

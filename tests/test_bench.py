@@ -108,3 +108,17 @@ def test_workload_selection_names_only_changes():
     args.flat_params = 1000
     wl = bench.select_workload(args)
     assert wl.d == 1000 and len(wl.tensors) == 1 and "flat tensor of 1000" in wl.name
+
+
+def test_clock_records_that_call_for_a_second_measurement():
+    """hw_slowdown, hw_thermal_slowdown and sw_thermal_slowdown reject a timed region, and so do SM clocks
+    well below their maximum with no reason given; sw_power_cap alone is kept."""
+    sys.path.insert(0, ROOT)
+    import bench
+    ok = {"reasons": [], "sm_mhz": 2070.0, "sm_max_mhz": 2070.0}
+    assert not bench.clocks_rejected(None) and not bench.clocks_rejected(ok)
+    assert not bench.clocks_rejected(dict(ok, reasons=["sw_power_cap"], sm_mhz=1750.0))
+    for reason in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
+        assert bench.clocks_rejected(dict(ok, reasons=[reason]))
+    assert bench.clocks_rejected(dict(ok, sm_mhz=1500.0))
+    assert bench.any_rank(True, 1) and not bench.any_rank(False, 1)
