@@ -427,8 +427,11 @@ const char* dsm_last_error(void);
  *
  * Arguments: layout, n (1..64) and hp as for dsm_create (the tensor list
  * passes the same checks; of hp only the global fields and the seed are
- * used, and global_mode must be DSM_GLOBAL_SIGN_MOMENTUM: the other global
- * steps return DSM_EINVAL here); gamma the round's gamma_t (> 0); round the
+ * used; global_mode is Algorithm 1's DSM_GLOBAL_SIGN_MOMENTUM or one of the
+ * variants that keep only x and m, DSM_GLOBAL_SLOWMO, _SIGNED_SLOWMO and
+ * _LOOKAHEAD, with m holding their momentum; DSM_GLOBAL_ADAMW, which also
+ * needs a second moment, returns DSM_EINVAL here, and so does a randomized
+ * sign_mode with a variant); gamma the round's gamma_t (> 0); round the
  * round index t (it keys the randomized sign); x and m the global model and
  * momentum (d fp32 each); replicas the n worker models (fp32, worker i at
  * replicas + i*replica_stride, replica_stride >= d and a multiple of 8);

@@ -163,8 +163,11 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     if (!(hp->g_eta >= 0.f && hp->g_eta < 3.0e38f) || !(hp->g_wd >= 0.f && hp->g_wd < 3.0e38f))
         return na_fail(DSM_EINVAL, "global eta and lambda must be finite and >= 0");
     if (hp->sign_mode < DSM_SIGN || hp->sign_mode > DSM_RSIGN_PM) return na_fail(DSM_EINVAL, "sign mode unknown");
-    if (hp->global_mode != DSM_GLOBAL_SIGN_MOMENTUM)
-        return na_fail(DSM_EINVAL, "only the sign-momentum global step (DSM_GLOBAL_SIGN_MOMENTUM) is available here");
+    if (hp->global_mode < DSM_GLOBAL_SIGN_MOMENTUM || hp->global_mode > DSM_GLOBAL_LOOKAHEAD)
+        return na_fail(DSM_EINVAL, "global step must be DSM_GLOBAL_SIGN_MOMENTUM, _SLOWMO, _SIGNED_SLOWMO or "
+                                   "_LOOKAHEAD here (global AdamW needs a second-moment buffer)");
+    if (hp->global_mode != DSM_GLOBAL_SIGN_MOMENTUM && hp->sign_mode != DSM_SIGN)
+        return na_fail(DSM_EINVAL, "the randomized signs apply to the sign-momentum global step only");
     if (hp->sign_mode != DSM_SIGN && !(hp->rsign_B > 0.f && hp->rsign_B < 3.0e38f))
         return na_fail(DSM_EINVAL, "randomized sign needs a finite bound B > 0");
     if (tiles > kNaMaxTiles)
@@ -216,7 +219,7 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     p.partials = reinterpret_cast<StatPartial*>(scratch + kOffPartials);
     p.stats = reinterpret_cast<TensorStats*>(scratch + kOffStats);
 
-    p.global_mode = DSM_GLOBAL_SIGN_MOMENTUM;
+    p.global_mode = hp->global_mode;
     LaunchShape ls;
     if ((err = query_launch_shape(p, &ls)) != cudaSuccess) return na_cuda(err, "occupancy query");
     GlobalScalars g{};
@@ -225,6 +228,9 @@ extern "C" int dsm_global_step_noalloc(const dsm_layout* layout, uint32_t n, con
     g.c1 = float((1.0 - double(hp->g_b1)) / double(gamma));
     g.c2 = float((1.0 - double(hp->g_b2)) / double(gamma));
     g.eta_gamma = float(double(hp->g_eta) * double(gamma));
+    g.inv_gamma = float(1.0 / double(gamma));
+    g.eta = hp->g_eta;
+    g.mode = hp->global_mode;
     g.B = hp->rsign_B;
     g.n_f = float(n);
     g.sign_mode = hp->sign_mode;

@@ -124,9 +124,9 @@ class LibraryWorkers:
       group.first_worker (dsm_set_first_worker), so that they draw the synthetic gradients of those
       workers of the n.
     - The owned range's global step is dsm_global_step_noalloc on the owner's x and m of the range and
-      the n models of the range (Algorithm 1's global step, the one that entry point runs), with the
-      range's layout placed at its first element (dsm_layout.first_element: the randomized sign's
-      counters are those of the whole model).
+      the n models of the range (Algorithm 1's global step, or the SlowMo, signed SlowMo and Lookahead
+      variants that entry point also runs), with the range's layout placed at its first element
+      (dsm_layout.first_element: the randomized sign's counters are those of the whole model).
     - The restart is dsm_end_round with the gathered x: the handle's workers start the next round from
       it, their base-optimizer states carry over.
     comm_device: where the collectives' tensors live ("cpu" for gloo, the CUDA device for NCCL)."""

@@ -36,6 +36,7 @@ CASES = {
     "adamw-fused-sign": dataclasses.replace(W.HParams(), flags=W.FLAG_FUSED_ROUND, seed=9),
     "sgdm-rsign0": dataclasses.replace(W.SGDM_HP, seed=2),
     "adamw-reset-local": dataclasses.replace(W.HParams(), flags=W.FLAG_RESET_LOCAL_STATE, seed=4),
+    "adamw-slowmo": dataclasses.replace(W.HParams(), global_mode=W.GLOBAL_SLOWMO, seed=7),
 }
 
 
@@ -140,8 +141,9 @@ def _rank_main(rank, world, port, case, n, tau, q):
 
 
 @pytest.mark.parametrize("case,n,world", [("adamw-bf16-rsignpm", 4, 2), ("sgdm-rsign0", 2, 2),
-                                          ("adamw-fused-sign", 3, 3)],
-                         ids=["adamw-n4-two-ranks", "sgdm-one-worker-per-rank", "fused-flag-three-ranks"])
+                                          ("adamw-fused-sign", 3, 3), ("adamw-slowmo", 4, 2)],
+                         ids=["adamw-n4-two-ranks", "sgdm-one-worker-per-rank", "fused-flag-three-ranks",
+                              "slowmo-two-ranks"])
 def test_worker_sharded_rounds_on_the_gpu_equal_one_process(dsm, case, n, world):
     tau = 2
     port = _free_port()

@@ -36,7 +36,12 @@ LARGE = (W.Tensor("big0", 3 * (1 << 20) + 5, W.KIND_WEIGHT, 1e-3), W.Tensor("big
 
 CASES = [("adamw-sign-n4", W.HParams(), 4, 2),
          ("sgdm-rsign-n3", dataclasses.replace(W.SGDM_HP, sign_mode=W.RSIGN_PM, rsign_B=1e-3), 3, 2),
-         ("adamw-rsign0-n9", dataclasses.replace(W.HParams(), sign_mode=W.RSIGN_ZERO, rsign_B=1.0), 9, 1)]
+         ("adamw-rsign0-n9", dataclasses.replace(W.HParams(), sign_mode=W.RSIGN_ZERO, rsign_B=1.0), 9, 1),
+         # the ablation global steps that keep only x and m
+         ("slowmo-n4", dataclasses.replace(W.HParams(), global_mode=W.GLOBAL_SLOWMO), 4, 2),
+         ("signed-slowmo-sgdm-n5", dataclasses.replace(W.SGDM_HP, sign_mode=W.SIGN,
+                                                       global_mode=W.GLOBAL_SIGNED_SLOWMO), 5, 1),
+         ("lookahead-n9", dataclasses.replace(W.HParams(), global_mode=W.GLOBAL_LOOKAHEAD), 9, 1)]
 
 
 def _need_gpu():
@@ -215,3 +220,18 @@ def test_noalloc_checks_every_buffer_and_the_tensor_list():
 
 def dsm_max_tiles():
     return 524288
+
+
+def test_noalloc_rejects_global_adamw_and_signed_variants_with_random_signs():
+    """Global AdamW needs a second-moment buffer this entry point does not take; the randomized signs belong
+    to Algorithm 1's global step only.  Both are refused before any work is enqueued."""
+    _need_gpu()
+    tensors = (W.Tensor("a", 64, W.KIND_WEIGHT, 1e-3),)
+    dev = torch.zeros(4 * 64, dtype=torch.float32, device="cuda")
+    for hp, what in ((dataclasses.replace(W.HParams(), global_mode=W.GLOBAL_ADAMW), "global AdamW"),
+                     (dataclasses.replace(W.HParams(), global_mode=W.GLOBAL_SLOWMO, sign_mode=W.RSIGN_ZERO,
+                                          rsign_B=1.0), "randomized signs")):
+        with pytest.raises(dsm.DsmError) as e:
+            dsm.dsm_global_step_noalloc(dsm.make_layout(tensors), 2, dsm.make_hparams(hp), 1e-3, 0,
+                                        dev.data_ptr(), dev.data_ptr(), dev.data_ptr(), 64)
+        assert e.value.code == dsm.DSM_EINVAL and what in str(e.value)
