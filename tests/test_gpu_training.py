@@ -8,7 +8,6 @@ comes from an autograd backward pass evaluated at that worker's model
 buffer (dsm_grad_ptr).  The oracle, fed the same gradients, must agree bit for
 bit, and the global model's loss over all classes must fall.
 """
-import dataclasses
 
 import numpy as np
 import pytest
