@@ -16,7 +16,8 @@ import workloads as W
 from gpu_common import compare_state
 
 torch = pytest.importorskip("torch")
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
 
 from oracle import dsm_oracle as O  # noqa: E402
 from paper_2411_17866_gb300 import dsm  # noqa: E402
