@@ -23,16 +23,35 @@ struct LocalItem {
     bool vec;
 };
 
+// A CTA's walk over the items: the (worker, tile) position of its current item, advanced by the grid
+// stride with one precomputed quotient and remainder instead of a division per item (the division by
+// the runtime tile count cost 0.4-0.7% of the local step on GPT-2 M and XL).
 template <bool kTileMajor>
-__device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t item, uint32_t e0, bool local_lam) {
-    uint32_t w, ti;
-    if (kTileMajor) {
-        ti = item / p.n;
-        w = item - ti * p.n;
-    } else {
-        w = item / p.num_tiles;
-        ti = item - w * p.num_tiles;
+struct ItemWalk {
+    uint32_t w, ti;        // position of the current item
+    uint32_t dq, dr;       // the stride as whole rows (tiles, or workers) and a remainder
+    __device__ __forceinline__ ItemWalk(const Problem& p, uint32_t item, uint32_t stride) {
+        const uint32_t row = kTileMajor ? p.n : p.num_tiles;  // items per row of the order
+        const uint32_t q = item / row, r = item - q * row;
+        if (kTileMajor) { ti = q; w = r; } else { w = q; ti = r; }
+        dq = stride / row;
+        dr = stride - dq * row;
     }
+    __device__ __forceinline__ void advance(const Problem& p) {
+        if (kTileMajor) {
+            ti += dq;
+            w += dr;
+            if (w >= p.n) { w -= p.n; ++ti; }
+        } else {
+            w += dq;
+            ti += dr;
+            if (ti >= p.num_tiles) { ti -= p.num_tiles; ++w; }
+        }
+    }
+};
+
+__device__ __forceinline__ LocalItem local_item(const Problem& p, uint32_t w, uint32_t ti, uint32_t e0,
+                                                bool local_lam) {
     const TileDesc td = p.tiles[ti];
     LocalItem it;
     it.base = w * p.d_stride + td.start;
@@ -53,7 +72,8 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
-    LocalItem nx = local_item<kFromGlobal>(p, item, e0, true);
+    ItemWalk<kFromGlobal> walk(p, item, gridDim.x);
+    LocalItem nx = local_item(p, walk.w, walk.ti, e0, true);
     float x[4], m[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f}, g[4];
     if (nx.vec) {
         load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
@@ -70,7 +90,8 @@ __global__ void __launch_bounds__(kThreads) k_local_adamw(Problem p, AdamScalars
         for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cm[j] = m[j]; cv[j] = v[j]; cg[j] = g[j]; }
         const uint32_t next = item + gridDim.x;
         if (next < items) {  // issue the next item's loads before computing this one
-            nx = local_item<kFromGlobal>(p, next, e0, true);
+            walk.advance(p);
+            nx = local_item(p, walk.w, walk.ti, e0, true);
             if (nx.vec) {
                 load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
                 if (!kZeroState) {
@@ -107,7 +128,8 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
     const uint32_t e0 = threadIdx.x * kElemsPerThread;
     uint32_t item = blockIdx.x;
     if (item >= items) return;
-    LocalItem nx = local_item<kFromGlobal>(p, item, e0, false);
+    ItemWalk<kFromGlobal> walk(p, item, gridDim.x);
+    LocalItem nx = local_item(p, walk.w, walk.ti, e0, false);
     float x[4], b[4] = {0.f, 0.f, 0.f, 0.f}, g[4];
     if (nx.vec) {
         load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
@@ -121,7 +143,8 @@ __global__ void __launch_bounds__(kThreads) k_local_sgdm(Problem p, SgdmScalars 
         for (int j = 0; j < 4; ++j) { cx[j] = x[j]; cb[j] = b[j]; cg[j] = g[j]; }
         const uint32_t next = item + gridDim.x;
         if (next < items) {
-            nx = local_item<kFromGlobal>(p, next, e0, false);
+            walk.advance(p);
+            nx = local_item(p, walk.w, walk.ti, e0, false);
             if (nx.vec) {
                 load4(kFromGlobal ? p.x + nx.start + e0 : p.X + nx.base + e0, x);
                 if (!kZeroState) load4(p.opt_m + nx.base + e0, b);
