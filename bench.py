@@ -42,8 +42,8 @@ import workloads as W  # noqa: E402
 METRIC = "params/s per global round (τ local + sign-momentum step); % HBM roofline"
 UNIT = "params/s"
 # the CPU oracle's samples: all host cores, and one thread (about 10-30 s of CPU work on the GPT-2 workloads)
-CPU_SAMPLE_ELEMS = 1 << 24
-CPU_ONE_CORE_ELEMS = 1 << 21
+CPU_SAMPLE_ELEMS = 1 << 27
+CPU_ONE_CORE_ELEMS = 1 << 24
 # the sources of the local-step kernels (their arithmetic lives in the shared device header)
 KERNELS_SRC = [os.path.join(ROOT, "paper_2411_17866_gb300", "csrc", f) for f in ("dsm_device.cuh", "dsm_local.cu")]
 
